@@ -1,0 +1,383 @@
+"""Benchmark of the routing-simulation hot path on GB300.
+
+One step = one pass of every hot-path row over one batch of synthetic input:
+  - the bursty replica sweep (4,096 replicas x 20,000 requests, 2 prefill + 6
+    decode instances, four policies): trace generation, simulation, goodput;
+  - the standalone scorer (2^20 requests x 64 instances).
+`value` is routed requests per second over the whole step (all ranks);
+scored pairs per second and per-kernel times are reported beside it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank simulates its own 4,096 replicas (replica offset
+rank * 4096; weak scaling, no collective on the data path).  --impl reference
+times the CPU oracle (the only reference this method has) on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import multiprocessing as mp
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_16206_gb300 import workloads as W  # noqa: E402
+
+N_SCORE_REQ = 1 << 20
+N_SCORE_INST = 64
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.samples = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 9:
+                self.samples.append(parts)
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = sorted(v for v in (num(s[1]) for s in self.samples) if v is not None)
+        mx = [v for v in (num(s[2]) for s in self.samples) if v is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for s in self.samples for i in range(4) if s[5 + i].lower() == "active"})
+        return {"sm_mhz": sm[len(sm) // 2] if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------- CPU oracle (baseline / reference arm)
+def _oracle_replica(args):
+    wl_name, replica, n_req, policies = args
+    import oracle
+    wl = {"replica_sweep": W.replica_sweep()}[wl_name]
+    tr = oracle.gen_trace(wl.trace, n_req, replica=replica)
+    routed = 0
+    for pol in policies:
+        res = oracle.simulate(wl.sim, W.CALIBRATED, pol, tr)
+        oracle.goodput(wl.sim, tr, res["t_first_us"], res["t_done_us"])
+        routed += n_req
+    return routed
+
+
+def oracle_rate(n_replicas: int, n_req: int, cores: int):
+    """Routed requests per second of the oracle over a replica sample, one
+    replica per process (spawned before any GPU work)."""
+    import oracle
+    oracle.build()
+    tasks = [("replica_sweep", r, n_req, list(W.ALL_POLICIES)) for r in range(n_replicas)]
+    ctx = mp.get_context("spawn")
+    t0 = time.perf_counter()
+    with ctx.Pool(processes=cores) as pool:
+        routed = sum(pool.map(_oracle_replica, tasks, chunksize=1))
+    dt = time.perf_counter() - t0
+    return routed / dt, routed, dt
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    cores = os.cpu_count() or 1
+    wl = W.replica_sweep()
+    n_rep = max(cores, 16)
+    for _ in range(args.warmup and 1):
+        oracle_rate(min(cores, 4), 2000, cores)
+    vals, walls = [], []
+    for _ in range(args.steps):
+        v, routed, dt = oracle_rate(n_rep, wl.n_req, cores)
+        vals.append(v)
+        walls.append(dt)
+    value = sum(vals) / len(vals)
+    sample = f"{n_rep} replicas x {wl.n_req} requests x 4 policies per step (of 4,096 replicas)"
+    line = {"impl": "reference", "metric": "routed requests/sec (replica sweep, 1 GB300)", "value": value,
+            "unit": "routed requests/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000 * sum(walls) / len(walls), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": wl.name, "replicas": wl.n_replicas, "requests_per_replica": wl.n_req,
+                       "pool": "2P+6D", "policies": 4, "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "routed requests/s", "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "routed requests/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------- GPU arm
+def _source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_16206_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def run_ours(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+
+    from paper_2609_16206_gb300 import build as ctr_build
+    if rank == 0:
+        ctr_build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    from paper_2609_16206_gb300 import ctr
+
+    cpu_base = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        n_rep = max(2 * cores, 16)
+        v, routed, dt = oracle_rate(n_rep, W.replica_sweep().n_req, cores)
+        cpu_base = {"value": v, "unit": "routed requests/s", "cores": cores, "kind": "oracle",
+                    "sample": f"{n_rep} replicas x 20000 requests x 4 policies, trace + simulation + goodput, "
+                              f"one replica per process ({dt:.1f} s wall)"}
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    wl = W.replica_sweep()
+    R, N = wl.n_replicas, wl.n_req
+    pols = list(W.ALL_POLICIES)
+    rows = R * len(pols)
+    offset = rank * R
+
+    tr = ctr.empty_requests(R, N, dev)
+    tf = torch.empty((rows, N), dtype=torch.int64, device=dev)
+    td = torch.empty_like(tf)
+    rhash = torch.empty(rows, dtype=torch.int64, device=dev)
+    rstat = torch.empty(rows, dtype=torch.int32, device=dev)
+    met = torch.empty(rows, dtype=torch.int64, device=dev)
+    p99 = torch.empty(rows, dtype=torch.int64, device=dev)
+    ws = ctr.simulate_workspace(wl.sim, rows, N, dev)
+    p, oh, cls = W.score_requests(N_SCORE_REQ, seed=0)
+    Q, A, kap = W.score_state(N_SCORE_INST, seed=1)
+    sp, soh, scls = (torch.from_numpy(x).to(dev) for x in (p, oh, cls))
+    sQ, sA, skap = (torch.from_numpy(x).to(dev) for x in (Q, A, kap))
+    sam = torch.empty(N_SCORE_REQ, dtype=torch.int32, device=dev)
+    scost = torch.empty(N_SCORE_REQ, dtype=torch.float32, device=dev)
+
+    ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(2)] for k in ("gen", "sim", "goodput", "score")}
+    times = {k: 0.0 for k in ev}
+
+    def step(timed: bool):
+        def mark(name, i):
+            if timed:
+                ev[name][i].record(stream)
+        mark("gen", 0)
+        ctr.ctr_gen_trace(wl.trace, R, offset, N, tr, stream=stream)
+        mark("gen", 1)
+        mark("sim", 0)
+        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, tr, R, N, tf, td, rhash, rstat, ws, stream=stream)
+        mark("sim", 1)
+        mark("goodput", 0)
+        ctr.ctr_goodput(wl.sim, tr, R, len(pols), N, tf, td, met, p99, stream=stream)
+        mark("goodput", 1)
+        mark("score", 0)
+        ctr.ctr_score_batch(sp, soh, scls, sQ, sA, skap, W.SCORE_CONSTS, sam, scost, stream=stream)
+        mark("score", 1)
+
+    def accumulate():
+        torch.cuda.synchronize()
+        for k, (a, b) in ev.items():
+            times[k] += a.elapsed_time(b)
+
+    for _ in range(args.warmup):
+        step(False)
+    torch.cuda.synchronize()
+    bad_rows = int((rstat != 0).sum())
+
+    clocks = ClockSampler(local_rank)
+    if rank == 0:
+        clocks.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        step(True)
+        accumulate()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop() if rank == 0 else None
+    ms_total = t0.elapsed_time(t1)
+    ms = torch.tensor([ms_total], dtype=torch.float64, device=dev)
+    if world > 1:
+        torch.distributed.all_reduce(ms, op=torch.distributed.ReduceOp.MAX)
+    ms_total = float(ms.item())
+    ms_step = ms_total / args.steps
+    routed_per_step = rows * N * world
+    value = routed_per_step / (ms_step / 1e3)
+    per_kernel_ms = {k: v / args.steps for k, v in times.items()}
+    pairs_per_s = N_SCORE_REQ * N_SCORE_INST / (per_kernel_ms["score"] / 1e3)
+
+    # ---- end to end through the public API with host buffers (rank-local)
+    host_tr = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in tr.items()}
+    for k in tr:
+        host_tr[k].copy_(tr[k])
+    host_score = [torch.from_numpy(x).pin_memory() for x in (p, oh, cls)]
+    out_host = {"met": torch.empty(rows, dtype=torch.int64, pin_memory=True),
+                "p99": torch.empty(rows, dtype=torch.int64, pin_memory=True),
+                "hash": torch.empty(rows, dtype=torch.int64, pin_memory=True),
+                "status": torch.empty(rows, dtype=torch.int32, pin_memory=True),
+                "am": torch.empty(N_SCORE_REQ, dtype=torch.int32, pin_memory=True),
+                "cost": torch.empty(N_SCORE_REQ, dtype=torch.float32, pin_memory=True)}
+    h2d = sum(v.numel() * v.element_size() for v in host_tr.values()) + sum(
+        v.numel() * v.element_size() for v in host_score)
+    d2h = sum(v.numel() * v.element_size() for v in out_host.values())
+
+    def e2e_step():
+        for k in tr:
+            tr[k].copy_(host_tr[k], non_blocking=True)
+        sp.copy_(host_score[0], non_blocking=True)
+        soh.copy_(host_score[1], non_blocking=True)
+        scls.copy_(host_score[2], non_blocking=True)
+        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, tr, R, N, tf, td, rhash, rstat, ws, stream=stream)
+        ctr.ctr_goodput(wl.sim, tr, R, len(pols), N, tf, td, met, p99, stream=stream)
+        ctr.ctr_score_batch(sp, soh, scls, sQ, sA, skap, W.SCORE_CONSTS, sam, scost, stream=stream)
+        out_host["met"].copy_(met, non_blocking=True)
+        out_host["p99"].copy_(p99, non_blocking=True)
+        out_host["hash"].copy_(rhash, non_blocking=True)
+        out_host["status"].copy_(rstat, non_blocking=True)
+        out_host["am"].copy_(sam, non_blocking=True)
+        out_host["cost"].copy_(scost, non_blocking=True)
+        torch.cuda.synchronize()
+
+    e2e_step()
+    e2e_steps = max(1, min(args.steps, 3))
+    if world > 1:
+        torch.distributed.barrier()
+    t_e0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    e2e_s = (time.perf_counter() - t_e0) / e2e_steps
+    e2e_t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+    if world > 1:
+        torch.distributed.all_reduce(e2e_t, op=torch.distributed.ReduceOp.MAX)
+    e2e_value = routed_per_step / float(e2e_t.item())
+
+    if rank != 0:
+        return 0
+    peaks = {}
+    pk_path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(pk_path):
+        with open(pk_path) as f:
+            peaks = json.load(f)
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
+    issue_peak = n_sm * 4 * sm_max * 1e6 / 1e9   # G warp-instructions / s
+    inst = SIM_INST_PER_LAUNCH.get(_source_hash())
+    sim_roof = {"bound": "alu", "unit": "Gwarp-inst/s", "peak": issue_peak,
+                "peak_source": f"{n_sm} SMs x 4 warp-inst/clk x {sm_max:.0f} MHz (max SM clock)",
+                "achieved": None, "frac": None, "traffic": None}
+    if inst is not None:
+        sim_roof["achieved"] = inst["warp_inst"] / (per_kernel_ms["sim"] / 1e3) / 1e9
+        sim_roof["frac"] = sim_roof["achieved"] / issue_peak
+        sim_roof["traffic"] = inst.get("dram_bytes")
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    score_bytes = 17 * N_SCORE_REQ + 3 * 4 * N_SCORE_INST
+    score_roof = {"bound": "hbm", "unit": "GB/s", "achieved": score_bytes / (per_kernel_ms["score"] / 1e3) / 1e9,
+                  "peak": hbm, "traffic": None}
+    score_roof["frac"] = score_roof["achieved"] / hbm
+    line = {
+        "metric": "routed requests/sec (replica sweep, 1 GB300)", "value": value, "unit": "routed requests/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic (seeded Philox traces shaped like the paper's mixed bursty workload)",
+        "config": {"workload": wl.name, "replicas_per_gpu": R, "requests_per_replica": N, "pool": "2P+6D",
+                   "policies": 4, "arrivals": "MMPP 3/12 req/s, 10 s mean dwell, seeds 0-2",
+                   "score_workload": f"{N_SCORE_REQ} requests x {N_SCORE_INST} instances",
+                   "l2": "inputs larger than L2 (1.7 GB trace, 5.2 GB of outputs per step)"},
+        "scored_pairs_per_s": pairs_per_s,
+        "kernel_ms": per_kernel_ms,
+        "rows_failed": bad_rows,
+        "roofline": sim_roof,
+        "roofline_score": score_roof,
+        "cpu_baseline": cpu_base,
+        "e2e": {"value": e2e_value, "unit": "routed requests/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h,
+                "note": "host trace + scorer inputs copied in, simulate + goodput + score, results copied out"},
+        "gpu_launches": 4 * args.steps,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# Executed warp instructions of one sim_kernel launch on the benchmarked
+# workload (ncu sm__inst_executed.sum), keyed by a hash of csrc/: a stale entry
+# (the kernel changed since the count was taken) reports null.
+SIM_INST_PER_LAUNCH: dict = {}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    try:
+        return run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,196 @@
+/*
+ * ctr.h -- C ABI of the GB300 marginal-cost routing simulator
+ * ("Calibrate, Then Route", arXiv 2609.16206).
+ *
+ * Exported by paper_2609_16206_gb300/libctr.so (CUDA, sm_103a).  Conventions
+ * for every entry point:
+ *   - Return 0 (CTR_OK) or a negative CTR_E* code.  Arguments are validated on
+ *     the host before any launch; a rejected call launches nothing.
+ *   - Arrays are DEVICE pointers owned by the caller unless marked "host".
+ *     The library allocates nothing and keeps no state between calls, so calls
+ *     on different streams are independent and thread-safe.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Work is enqueued asynchronously; nothing synchronises unless
+ *     stated.  Launch failures are reported as CTR_ECUDA.
+ *   - All simulated times are int64 microseconds.
+ */
+#ifndef CTR_H
+#define CTR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define CTR_OK 0
+#define CTR_EINVAL (-1)    /* bad argument, enum, bound or request data */
+#define CTR_ECUDA (-2)     /* CUDA launch / driver error */
+#define CTR_EOVERFLOW (-3) /* a fixed-capacity structure filled up, or a time reached 2^40 us */
+#define CTR_ETIMEOUT (-4)  /* the per-instance decode-step budget ran out */
+
+#define CTR_MAX_INSTANCES 32      /* prefill + decode instances of one simulated cluster */
+#define CTR_MAX_CLASSES 4         /* SLO classes */
+#define CTR_MAX_CONST_SETS 128    /* cost-constant sets per ctr_simulate call */
+#define CTR_MAX_REQUESTS (1 << 23) /* requests per replica */
+#define CTR_SCORE_N_CONST 13      /* length of the standalone scorer's constant vector */
+#define CTR_SCORE_MAX_INST 256    /* instances per standalone scoring call */
+
+enum ctr_policy {
+    CTR_POLICY_LEARNED = 0,          /* marginal-cost argmin, sec. III-A / Algorithm 1 */
+    CTR_POLICY_ROUND_ROBIN = 1,      /* request k -> instance k mod N, sec. IV-C */
+    CTR_POLICY_LEAST_LOADED = 2,     /* argmin of in-flight count (JSQ), sec. IV-C */
+    CTR_POLICY_LENGTH_HEURISTIC = 3  /* predicted-length threshold heuristic, sec. IV-C */
+};
+
+enum ctr_workspace_kind { CTR_WS_SIMULATE = 0 };
+
+/* A batch of requests in structure-of-arrays form: element [r * n_req + k] is
+ * request k (0-based arrival index) of replica r.  Device memory, caller-owned.
+ * The request features are the four admission-time signals of sec. III-A:
+ * exact prompt length p, predicted output length o_hat, SLO class, plus the
+ * true output length o (known to the simulated cluster only) and the arrival. */
+typedef struct ctr_requests {
+    int64_t* arrival_us; /* non-decreasing within a replica, < 2^39 */
+    int32_t* prompt_len; /* p, 0..2^20 */
+    int32_t* true_out;   /* o, 1..2^20, p + o <= kv_cap_tokens */
+    int32_t* pred_out;   /* o_hat, 0..2^17 */
+    uint8_t* slo_class;  /* 0..n_classes-1 */
+} ctr_requests;
+
+/* Synthetic trace law (a host struct).  Replica g (global index) draws from the
+ * Philox4x32-10 key seed + (g mod n_seeds), sub-stream g / n_seeds; counter
+ * (k, sub, stream, group).  Lengths are rounded lognormals, o_hat = o * exp(N(0,
+ * noise_sigma)) rounded, class from cumulative 32-bit thresholds, arrivals the
+ * integer Poisson (arrival_kind 0) or two-state MMPP (1, low state first)
+ * construction.  All doubles must be finite. */
+typedef struct ctr_trace_cfg {
+    uint64_t seed;
+    int32_t n_seeds;          /* >= 1 */
+    int32_t arrival_kind;     /* 0 Poisson at rate_mreq[0]; 1 MMPP rate_mreq[0] / [1] */
+    int64_t rate_mreq[2];     /* milli-requests per second, 1..10^7 */
+    int64_t dwell_mean_us;    /* MMPP mean state dwell, 1..10^10 */
+    double prompt_mu, prompt_sigma;   /* ln-space mean / sd of the prompt length */
+    int32_t prompt_min, prompt_max;   /* clip range, 0 <= min <= max <= 2^20 */
+    uint64_t mix_short_thr;           /* P(short output component) * 2^32, <= 2^32 */
+    double short_mu, short_sigma, long_mu, long_sigma;
+    int32_t out_min, out_max;         /* 1 <= min <= max <= 2^20 */
+    double noise_sigma;               /* predictor noise, >= 0 */
+    int32_t pred_min, pred_max;       /* 0 <= min <= max <= 2^17 */
+    int32_t n_classes;                /* 1..4 */
+    int32_t reserved0;
+    uint64_t class_thr[3];            /* cumulative class probabilities * 2^32, non-decreasing */
+} ctr_trace_cfg;
+
+/* Simulated cluster (a host struct): explicit prefill and decode pools, KV
+ * transfer, continuous decode batching with KV reservation, SLO classes, and
+ * the capacities of the per-instance structures the GPU keeps. */
+typedef struct ctr_sim_cfg {
+    int32_t n_prefill, n_decode;      /* >= 1 each, n_prefill + n_decode <= 32 */
+    int64_t kv_cap_tokens;            /* C per decode instance, 1..2^31-1 */
+    int64_t pre_base_us;              /* prefill = base + per_tok * p; base 1..2^30 */
+    int64_t pre_us_per_tok;           /* 0..2^20 */
+    int64_t xfer_us_per_tok;          /* KV transfer delay = per_tok * p; 0..2^20 */
+    int64_t dec_base_us;              /* decode step = base + per_seq * n + floor(KV / kv_div); base 1..2^24 */
+    int64_t dec_us_per_seq;           /* 0..2^16 */
+    int64_t dec_kv_tokens_per_us;     /* kv_div, 1..2^31 */
+    int32_t n_classes;                /* 1..4 */
+    int32_t heuristic_threshold_tokens; /* length heuristic: o_hat >= threshold uses predicted-token load */
+    int64_t ttft_slo_us[4];           /* per class, >= 0 */
+    int64_t tpot_slo_us[4];
+    int64_t max_steps_per_instance;   /* decode-step budget per instance and row, >= 1 */
+    int32_t cap_pending;              /* requests routed to a decode instance whose KV is not ready, 1..2^20 */
+    int32_t cap_waiting;              /* KV-ready requests not yet admitted, 1..2^20 */
+    int32_t cap_active;               /* decode batch size, 1..2^20 */
+    int32_t cap_prefill_ring;         /* requests in flight on a prefill instance, 1..2^20 */
+} ctr_sim_cfg;
+
+/* Fixed-point constants of the learned router (a host struct).  Weights carry
+ * 8 fractional bits (256 = 1.0).  Decode cost, in us * 2^16:
+ *   P     = min(2^18, floor((KV_res + p + o_hat) * 2^16 / C))     post-admission pressure
+ *   own   = o_hat * tau_dec
+ *   T2    = own + floor(floor(own * P / 2^16) * rho / 2^8)
+ *   cost  = (w_b * min(B_d, 2^40) + w_s * T2) * sigma[class] + w_q * queue * 2^16
+ * Prefill cost: (w_b * B_p + w_s * (tau_pre0 + p * tau_pre)) * sigma[class] + w_q * queue * 2^16,
+ * with backlog B_p = max(0, busy_until - t) and B_d = floor(R_d * step_d / max(1, n_d)). */
+typedef struct ctr_cost_consts {
+    int64_t tau_pre0_us, tau_pre_us, tau_dec_us; /* 0..2^20 */
+    int64_t w_q_us;                              /* 0..2^20, us per in-flight request */
+    int32_t w_b_q8, w_s_q8, rho_q8;              /* 0..1023 */
+    int32_t sigma_q8[4];                         /* 0..1023 */
+    int32_t reserved0;
+} ctr_cost_consts;
+
+/* ctr_gen_trace -- synthetic request trace (Table 1 length profiles as
+ * lognormal laws; the sec. III-C predictor with sec. V-G injected noise;
+ * bursty arrivals).  Fills out[r * n_req + k] for replicas
+ * g = replica_offset + r, r < n_replicas.  The result is bit-identical to the
+ * CPU reference construction (deterministic fp64, integer arrivals).
+ * n_req 0..CTR_MAX_REQUESTS; n_replicas >= 0; replica_offset >= 0. */
+int ctr_gen_trace(const ctr_trace_cfg* cfg /* host */, int32_t n_replicas, int64_t replica_offset,
+                  int64_t n_req, ctr_requests out, void* stream);
+
+/* ctr_score_batch -- standalone marginal-cost scorer (sec. III-A display) of
+ * every request x instance pair over a mixed per-instance state: queued
+ * prefill tokens Q, active decode sequences A, KV occupancy kappa.
+ *   cost(r,d) = sigma_s * (w_b * (tau_pre Q_d + tau_act A_d)
+ *               + w_s * (tau_pre0 + tau_pre p + tau_dec o_hat (1 + rho (kappa_d + (p + o_hat) / C))))
+ *               + w_q A_d
+ * consts (host, CTR_SCORE_N_CONST floats, finite, >= 0):
+ *   [w_b, w_s, w_q, rho, tau_pre0, tau_pre, tau_dec, tau_act, 1/C, sigma_0..sigma_3].
+ * Per request r: out_argmin[r] = argmin_d (ties -> lowest d) and out_cost[r]
+ * its fp32 cost; a slo_class >= 4 gives -1 and NaN.  Inputs must be finite and
+ * non-negative.  n_req >= 0, 1 <= n_inst <= CTR_SCORE_MAX_INST.  status is an
+ * optional device int32 (NULL ok) set to CTR_ETIMEOUT if the shared-memory
+ * staging wait of a block ran past its bound (never expected). */
+int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_t* slo_class, int64_t n_req,
+                    const float* q_tokens, const float* n_active, const float* kv_occ, int32_t n_inst,
+                    const float* consts /* host */, int32_t* out_argmin, float* out_cost, int32_t* status,
+                    void* stream);
+
+/* ctr_workspace_bytes -- device workspace ctr_simulate needs to run its
+ * widest grid for these sizes on the current device (0 on bad arguments).
+ * A smaller workspace is accepted and runs fewer concurrent rows. */
+size_t ctr_workspace_bytes(int32_t which, const ctr_sim_cfg* cfg /* host */, int64_t n_rows, int64_t n_req);
+
+/* ctr_simulate -- batched discrete-event simulation of the routing policies
+ * (Algorithm 1 inside the sec. III-D simulator with sec. VI batching).
+ * Rows are (replica, const set, policy), row-major:
+ *   row = (replica * n_const_sets + set) * n_policies + policy_index.
+ * Replica r reads trace[r * n_req + k]; outputs are [row * n_req + k].
+ * consts: n_const_sets host structs (1..CTR_MAX_CONST_SETS); policy_ids:
+ * n_policies host ints (1..4), values of enum ctr_policy.
+ * Outputs: i_pre / i_dec (optional, NULL ok) chosen prefill / decode instance;
+ * t_first_us (end of the first decode step) and t_done_us (required);
+ * row_hash the order-independent 64-bit checksum of each row's routing and
+ * times; row_status CTR_OK or the row's CTR_EINVAL / CTR_EOVERFLOW /
+ * CTR_ETIMEOUT (outputs of a failed row are unspecified).
+ * workspace: device, >= 256 bytes, ideally ctr_workspace_bytes(); its contents
+ * need no initialisation and are clobbered. */
+int ctr_simulate(const ctr_sim_cfg* cfg /* host */, const ctr_cost_consts* consts /* host */, int32_t n_const_sets,
+                 const int32_t* policy_ids /* host */, int32_t n_policies, ctr_requests trace, int32_t n_replicas,
+                 int64_t n_req, uint8_t* i_pre, uint8_t* i_dec, int64_t* t_first_us, int64_t* t_done_us,
+                 uint64_t* row_hash, int32_t* row_status, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ctr_goodput -- SLO goodput inputs per row (sec. IV-B targets, Table 2
+ * columns): met_count[row] = #{k : TTFT <= TTFT_c and (o == 1 or
+ * t_done - t_first <= TPOT_c (o - 1))} and p99_ttft_us[row] = the nearest-rank
+ * P99 (sorted index ceil(0.99 n) - 1; -1 when n_req == 0).  Row r uses replica
+ * r / rows_per_replica of the trace.  A class >= n_classes counts as the last
+ * class. */
+int ctr_goodput(const ctr_sim_cfg* cfg /* host */, ctr_requests trace, int32_t n_replicas, int32_t rows_per_replica,
+                int64_t n_req, const int64_t* t_first_us, const int64_t* t_done_us, int64_t* met_count,
+                int64_t* p99_ttft_us, void* stream);
+
+/* ctr_strerror -- static description of a CTR_* code. */
+const char* ctr_strerror(int code);
+
+/* ctr_abi_version -- increments on any change to the structs or signatures. */
+int ctr_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CTR_H */

@@ -1,0 +1,106 @@
+// ctr_internal.cuh -- declarations shared by the CUDA translation units of
+// libctr.so (kernel parameter blocks and launchers).  Not part of the ABI.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/ctr.h"
+
+namespace ctr {
+
+constexpr int kWarp = 32;
+constexpr int64_t kTimeLimit = int64_t(1) << 40;   // every simulated time stays below this
+constexpr int64_t kArrivalLimit = int64_t(1) << 39;
+constexpr int kKeyBits = 23;                        // request index bits in packed heap keys
+constexpr uint64_t kKeyMask = (uint64_t(1) << kKeyBits) - 1;
+
+// ---------------------------------------------------------------- trace
+struct TraceParams {
+    uint64_t seed;
+    int64_t n_seeds;
+    int32_t arrival_kind;
+    int32_t n_classes;
+    int64_t rate[2];
+    int64_t dwell_mean_us;
+    double prompt_mu, prompt_sigma, short_mu, short_sigma, long_mu, long_sigma, noise_sigma;
+    int64_t prompt_min, prompt_max, out_min, out_max, pred_min, pred_max;
+    uint64_t mix_short_thr;
+    uint64_t class_thr[3];
+    int64_t n_replicas, replica_offset, n_req;
+    ctr_requests out;
+};
+cudaError_t launch_trace(const TraceParams& p, cudaStream_t stream);
+
+// ---------------------------------------------------------------- simulator
+struct ConstsDev {
+    int64_t tau_pre0, tau_pre, tau_dec, w_q;
+    int32_t w_b, w_s, rho, sigma[4];
+    int32_t pad;
+};
+
+struct SimParams {
+    int32_t n_pre, n_dec;
+    int64_t kv_cap;
+    uint64_t kv_cap_recip;      // floor((2^64 - 1) / kv_cap)
+    int64_t pre_base, pre_tok, xfer_tok;
+    int64_t dec_base, dec_seq;
+    int64_t kv_div;
+    uint64_t kv_div_magic;      // ceil(2^64 / kv_div) (kv_div >= 2)
+    int32_t n_classes, heur_thresh;
+    int64_t max_steps;
+    int32_t cap_pend, cap_wait, cap_act, cap_ring;
+    int32_t n_sets, n_pols;
+    int32_t pols[4];
+    int64_t n_req, n_rows;
+    // per-slot workspace: interleaved [entry][lane] arrays
+    unsigned char* ws;
+    uint32_t* next_row;
+    int64_t slot_bytes;
+    int64_t off_act, off_wait;  // byte offsets of the active heap and waiting ring inside a slot
+    int32_t cap_pr;             // max(cap_pend, cap_ring): entries of the first region
+    int32_t n_slots;
+    ctr_requests trace;
+    uint8_t* i_pre;
+    uint8_t* i_dec;
+    int64_t* t_first;
+    int64_t* t_done;
+    uint64_t* row_hash;
+    int32_t* row_status;
+    ConstsDev sets[CTR_MAX_CONST_SETS];
+};
+int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr);
+int sim_max_resident_warps(int* warps_per_block, int* blocks);
+cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream);
+
+// ---------------------------------------------------------------- goodput
+struct GoodputParams {
+    ctr_requests trace;
+    int64_t n_req, n_rows;
+    int32_t rows_per_replica, n_classes;
+    int64_t ttft[4], tpot[4];
+    const int64_t* t_first;
+    const int64_t* t_done;
+    int64_t* met;
+    int64_t* p99;
+};
+cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream);
+
+// ---------------------------------------------------------------- standalone scorer
+struct ScoreParams {
+    const float* p;
+    const float* oh;
+    const uint8_t* cls;
+    int64_t n;
+    const float* Q;
+    const float* A;
+    const float* kap;
+    int32_t n_inst;
+    float c[CTR_SCORE_N_CONST];
+    int32_t* argmin;
+    float* cost;
+    int32_t* status;
+};
+cudaError_t launch_score(const ScoreParams& p, cudaStream_t stream);
+
+}  // namespace ctr

@@ -1,0 +1,148 @@
+// goodput.cu -- SLO goodput inputs per simulated row (ctr_goodput):
+// the count of requests meeting both SLOs of their class (sec. IV-B targets,
+// Table 2 goodput) and the exact nearest-rank P99 TTFT (Table 2 column).
+//
+// One 256-thread block per row.  Pass 0 reads the row once and reduces the
+// met count and the TTFT range; the P99 is then selected exactly by a radix
+// select over (TTFT - min) with 11-bit digits, most significant first, each
+// pass histogramming the candidates that still match the digits chosen so far
+// (2048 shared-memory bins).  Rows are re-read from L2 by each pass.
+#include "ctr_internal.cuh"
+
+namespace ctr {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kDigit = 11;
+constexpr int kBins = 1 << kDigit;
+
+template <typename T, typename Op>
+__device__ T block_reduce(T v, T identity, Op op, T* scratch)
+{
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) v = op(v, __shfl_xor_sync(0xffffffffu, v, off));
+    if (lane == 0) scratch[wid] = v;
+    __syncthreads();
+    if (wid == 0) {
+        v = lane < kThreads / 32 ? scratch[lane] : identity;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) v = op(v, __shfl_xor_sync(0xffffffffu, v, off));
+        if (lane == 0) scratch[0] = v;
+    }
+    __syncthreads();
+    const T r = scratch[0];
+    __syncthreads();
+    return r;
+}
+
+__global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P)
+{
+    __shared__ uint32_t hist[kBins];
+    __shared__ int64_t red64[kThreads / 32];
+    __shared__ uint32_t pick[2];
+    const int tid = threadIdx.x;
+    const int64_t n = P.n_req;
+
+    for (int64_t row = blockIdx.x; row < P.n_rows; row += gridDim.x) {
+        const int64_t tb = (row / P.rows_per_replica) * n;
+        const int64_t ob = row * n;
+        int64_t met = 0, mn = INT64_MAX, mx = INT64_MIN;
+        for (int64_t k = tid; k < n; k += kThreads) {
+            const int64_t tf = P.t_first[ob + k];
+            const int64_t td = P.t_done[ob + k];
+            const int64_t ttft = tf - P.trace.arrival_us[tb + k];
+            const int64_t o = P.trace.true_out[tb + k];
+            int c = P.trace.slo_class[tb + k];
+            if (c >= P.n_classes) c = P.n_classes - 1;
+            const bool ok = ttft <= P.ttft[c] && (o == 1 || td - tf <= P.tpot[c] * (o - 1));
+            met += ok;
+            mn = ttft < mn ? ttft : mn;
+            mx = ttft > mx ? ttft : mx;
+        }
+        met = block_reduce<int64_t>(met, 0, [](int64_t a, int64_t b) { return a + b; }, red64);
+        mn = block_reduce<int64_t>(mn, INT64_MAX, [](int64_t a, int64_t b) { return a < b ? a : b; }, red64);
+        mx = block_reduce<int64_t>(mx, INT64_MIN, [](int64_t a, int64_t b) { return a > b ? a : b; }, red64);
+        if (n == 0) {
+            if (tid == 0) {
+                P.met[row] = 0;
+                P.p99[row] = -1;
+            }
+            continue;
+        }
+        const uint64_t range = (uint64_t)mx - (uint64_t)mn;
+        int shift = range == 0 ? 0 : 64 - __clzll((long long)range);  // bits still undetermined
+        uint64_t prefix = 0;                                            // chosen high bits of (ttft - mn)
+        int64_t rank = (99 * n + 99) / 100 - 1;                         // 0-based rank among the candidates
+        while (shift > 0) {
+            const int dbits = shift < kDigit ? shift : kDigit;
+            const int above = shift;  // candidates agree with prefix on bits >= above
+            shift -= dbits;
+            for (int i = tid; i < kBins; i += kThreads) hist[i] = 0;
+            __syncthreads();
+            const uint32_t dmask = (1u << dbits) - 1u;
+            for (int64_t k = tid; k < n; k += kThreads) {
+                const uint64_t v = (uint64_t)(P.t_first[ob + k] - P.trace.arrival_us[tb + k]) - (uint64_t)mn;
+                const bool match = above >= 64 || (v >> above) == (prefix >> above);
+                if (match) atomicAdd(&hist[(uint32_t)(v >> shift) & dmask], 1u);
+            }
+            __syncthreads();
+            if (tid < 32) {  // find the bin holding the rank: per-lane sums, then a scan
+                const int per = kBins / 32;
+                uint32_t sum = 0;
+                for (int i = 0; i < per; ++i) sum += hist[tid * per + i];
+                uint32_t incl = sum;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const uint32_t v = __shfl_up_sync(0xffffffffu, incl, off);
+                    if (tid >= off) incl += v;
+                }
+                const uint32_t excl = incl - sum;
+                const bool mine = (int64_t)excl <= rank && rank < (int64_t)incl;
+                const uint32_t ball = __ballot_sync(0xffffffffu, mine);
+                const int owner = __ffs(ball) - 1;
+                if (tid == owner) {
+                    uint32_t acc = excl;
+                    int bin = tid * per;
+                    for (int i = 0; i < per; ++i) {
+                        const uint32_t hcount = hist[tid * per + i];
+                        if ((int64_t)(acc + hcount) > rank) {
+                            bin = tid * per + i;
+                            break;
+                        }
+                        acc += hcount;
+                    }
+                    pick[0] = (uint32_t)bin;
+                    pick[1] = acc;
+                }
+            }
+            __syncthreads();
+            prefix |= (uint64_t)pick[0] << shift;
+            rank -= pick[1];
+            __syncthreads();
+        }
+        if (tid == 0) {
+            P.met[row] = met;
+            P.p99[row] = (int64_t)((uint64_t)mn + prefix);
+        }
+        __syncthreads();
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream)
+{
+    if (p.n_rows == 0) return cudaSuccess;
+    int dev = 0, sms = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    int64_t blocks = p.n_rows;
+    if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
+    goodput_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace ctr

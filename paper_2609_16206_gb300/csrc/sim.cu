@@ -1,0 +1,450 @@
+// sim.cu -- batched discrete-event simulation of request routing
+// (ctr_simulate): Algorithm 1 of the paper inside the sec. III-D simulator,
+// with the continuous decode batching of sec. VI, the marginal-cost score of
+// sec. III-A and the sec. IV-C baselines.
+//
+// Layout: one warp simulates one row (replica x cost-constant set x policy);
+// lane i < n_pre is prefill instance i, lane n_pre + d is decode instance d.
+// Warps are persistent and pull rows from an atomic counter in the workspace,
+// so rows of different length balance across the GPU.  For every arrival k:
+//   1. each decode lane advances its own instance's event loop to t_k
+//      (step ends, KV-ready events, FCFS admissions, step starts);
+//      each prefill lane retires prefills that ended by t_k;
+//   2. every lane prices its instance for the policy, and two warp-wide
+//      argmins (redux.sync, ties to the lowest lane) pick i_pre and i_dec;
+//   3. the i_pre lane commits the FCFS prefill, broadcasts the KV-ready time,
+//      and the i_dec lane queues the request.
+// All time and cost arithmetic is int64 fixed point, so every decision is
+// deterministic.  Instances never interact except through routing, so the
+// per-lane event loops reproduce the global event order exactly (events at
+// an arrival's own time are processed before it is routed).
+//
+// Per-lane structures live in the workspace slot of the warp, interleaved
+// [entry][lane] so that the lanes' heap tops share cache lines: a min-heap of
+// pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
+// lanes use the same region as their in-flight ring of prefill end times),
+// a min-heap of active requests keyed by finishing step (finish << 23 | k),
+// and a FIFO ring of KV-ready requests awaiting admission.  Heap tops are
+// cached in registers, so a plain decode step touches no memory.
+#include "ctr_internal.cuh"
+
+namespace ctr {
+namespace {
+
+constexpr uint64_t kEmpty = ~0ull;
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kWarpsPerBlock = 4;
+constexpr int64_t kNever = INT64_MAX;
+constexpr int64_t kBacklogClamp = int64_t(1) << 40;
+constexpr int64_t kPressureClamp = int64_t(1) << 18;
+
+__device__ __forceinline__ uint64_t mix64(uint64_t z)  // splitmix64 output function
+{
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ uint64_t hterm(int64_t k, uint64_t tag, uint64_t v)
+{
+    return mix64(mix64((tag << 56) ^ (uint64_t)k) ^ v);
+}
+
+// floor(num / d) with r = floor((2^64 - 1) / d): the estimate is low by at most 2
+__device__ __forceinline__ uint64_t div_recip(uint64_t num, uint64_t d, uint64_t recip)
+{
+    uint64_t q = __umul64hi(num, recip);
+    uint64_t r = num - q * d;
+    if (r >= d) {
+        ++q;
+        r -= d;
+    }
+    if (r >= d) ++q;
+    return q;
+}
+
+// floor(x / kv_div) for 0 <= x < 2^32 with magic = ceil(2^64 / kv_div), exact
+__device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
+{
+    return P.kv_div == 1 ? x : (int64_t)__umul64hi((uint64_t)x, P.kv_div_magic);
+}
+
+// min-heap of unique 64-bit keys with stride-32 (interleaved) storage
+__device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
+{
+    int i = n++;
+    while (i > 0) {
+        const int parent = (i - 1) >> 1;
+        const uint64_t pv = h[parent * kWarp];
+        if (pv < key) break;
+        h[i * kWarp] = pv;
+        i = parent;
+    }
+    h[i * kWarp] = key;
+    if (i == 0) top = key;
+}
+
+__device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
+{
+    const int m = --n;
+    if (m == 0) {
+        top = kEmpty;
+        return;
+    }
+    const uint64_t last = h[m * kWarp];
+    int i = 0;
+    for (;;) {
+        int c = 2 * i + 1;
+        if (c >= m) break;
+        uint64_t cv = h[c * kWarp];
+        if (c + 1 < m) {
+            const uint64_t rv = h[(c + 1) * kWarp];
+            if (rv < cv) {
+                cv = rv;
+                ++c;
+            }
+        }
+        if (last < cv) break;
+        h[i * kWarp] = cv;
+        i = c;
+    }
+    h[i * kWarp] = last;
+    top = h[0];
+}
+
+// argmin over the lanes of 64-bit values (ties -> lowest lane)
+__device__ __forceinline__ int warp_argmin(uint64_t v)
+{
+    const uint32_t hi = (uint32_t)(v >> 32), lo = (uint32_t)v;
+    const uint32_t mhi = __reduce_min_sync(kFull, hi);
+    const uint32_t mlo = __reduce_min_sync(kFull, hi == mhi ? lo : 0xffffffffu);
+    const uint32_t ball = __ballot_sync(kFull, hi == mhi && lo == mlo);
+    return __ffs(ball) - 1;
+}
+
+struct Decode {
+    int64_t step_end, step_idx, kv_res, kv_rsv, R, ohat, steps;
+    uint64_t pend_top, act_top;
+    int32_t n_act, q, pend_n, act_n, w_head, w_n;
+    bool stepping;
+};
+
+// Advance one decode instance through every event at times <= T.
+__device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
+                                              uint32_t* wait, int64_t tb, int64_t ob, uint64_t& h)
+{
+    for (;;) {
+        const int64_t te = s.stepping ? s.step_end : kNever;
+        const int64_t tp = s.pend_n > 0 ? (int64_t)(s.pend_top >> kKeyBits) : kNever;
+        const int64_t tev = te < tp ? te : tp;
+        if (tev > T) return CTR_OK;
+        if (te == tev) {  // (1) the running step ends: one token for every active request
+            s.step_idx += 1;
+            s.kv_res += s.n_act;
+            s.R -= s.n_act;
+            s.stepping = false;
+            while (s.act_n > 0 && (int64_t)(s.act_top >> kKeyBits) == s.step_idx) {
+                const int64_t k = (int64_t)(s.act_top & kKeyMask);
+                heap_pop(act, s.act_n, s.act_top);
+                const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
+                const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
+                const int64_t ohk = __ldg(&P.trace.pred_out[tb + k]);
+                s.n_act -= 1;
+                s.q -= 1;
+                s.kv_res -= pk + ok;
+                s.kv_rsv -= pk + ok;
+                s.ohat -= ohk;
+                P.t_done[ob + k] = tev;
+                h += hterm(k, 3, (uint64_t)tev);
+            }
+        }
+        // (2) KV-ready requests join the waiting FIFO in (time, index) order
+        while (s.pend_n > 0 && (int64_t)(s.pend_top >> kKeyBits) == tev) {
+            const uint32_t k = (uint32_t)(s.pend_top & kKeyMask);
+            heap_pop(pend, s.pend_n, s.pend_top);
+            if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
+            int pos = s.w_head + s.w_n;
+            if (pos >= P.cap_wait) pos -= P.cap_wait;
+            wait[pos * kWarp] = k;
+            s.w_n += 1;
+        }
+        // (3) not mid-step: strict FCFS admission while the reservation fits, then start a step
+        if (!s.stepping) {
+            const int pos0 = s.w_head;
+            int admitted = 0;
+            while (s.w_n > 0) {
+                const uint32_t k = wait[s.w_head * kWarp];
+                const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
+                const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
+                if (s.kv_rsv + pk + ok > P.kv_cap) break;
+                if (s.act_n == P.cap_act) return CTR_EOVERFLOW;
+                s.w_head = s.w_head + 1 == P.cap_wait ? 0 : s.w_head + 1;
+                s.w_n -= 1;
+                s.kv_rsv += pk + ok;
+                s.kv_res += pk;
+                s.n_act += 1;
+                heap_push(act, s.act_n, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
+                admitted += 1;
+            }
+            if (s.n_act > 0) {
+                if (++s.steps > P.max_steps) return CTR_ETIMEOUT;
+                s.step_end = tev + P.dec_base + P.dec_seq * s.n_act + kv_term(s.kv_res, P);
+                if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
+                s.stepping = true;
+                int pos = pos0;
+                for (int i = 0; i < admitted; ++i) {  // first token at the end of this step
+                    const uint32_t k = wait[pos * kWarp];
+                    P.t_first[ob + k] = s.step_end;
+                    h += hterm(k, 2, (uint64_t)s.step_end);
+                    pos = pos + 1 == P.cap_wait ? 0 : pos + 1;
+                }
+            }
+        }
+    }
+}
+
+// Per-request bounds, arrival order (CTR_EINVAL before anything is simulated).
+__device__ __forceinline__ bool row_valid(const SimParams& P, int64_t tb, int lane)
+{
+    int64_t prev_last = 0;
+    for (int64_t base = 0; base < P.n_req; base += 32) {
+        const int64_t k = base + lane;
+        const bool live = k < P.n_req;
+        int64_t t = 0;
+        bool bad = false;
+        if (live) {
+            t = P.trace.arrival_us[tb + k];
+            const int64_t p = P.trace.prompt_len[tb + k];
+            const int64_t o = P.trace.true_out[tb + k];
+            const int64_t oh = P.trace.pred_out[tb + k];
+            const int64_t c = P.trace.slo_class[tb + k];
+            bad = t < 0 || t >= kArrivalLimit || p < 0 || p > (1 << 20) || o < 1 || o > (1 << 20) ||
+                  p + o > P.kv_cap || oh < 0 || oh > (1 << 17) || c >= P.n_classes;
+        }
+        int64_t before = __shfl_up_sync(kFull, t, 1);
+        if (lane == 0) before = prev_last;
+        if (live && t < before) bad = true;
+        if (__any_sync(kFull, bad)) return false;
+        prev_last = __shfl_sync(kFull, t, 31);
+    }
+    return true;
+}
+
+__global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_constant__ SimParams P)
+{
+    const int lane = threadIdx.x & 31;
+    const int64_t slot = (int64_t)blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
+    if (slot >= P.n_slots) return;
+    unsigned char* sb = P.ws + slot * P.slot_bytes;
+    uint64_t* pend = reinterpret_cast<uint64_t*>(sb) + lane;
+    int64_t* ring = reinterpret_cast<int64_t*>(sb) + lane;
+    uint64_t* act = reinterpret_cast<uint64_t*>(sb + P.off_act) + lane;
+    uint32_t* wait = reinterpret_cast<uint32_t*>(sb + P.off_wait) + lane;
+
+    const bool is_pre = lane < P.n_pre;
+    const bool is_dec = lane >= P.n_pre && lane < P.n_pre + P.n_dec;
+    const int64_t per_rep = (int64_t)P.n_sets * P.n_pols;
+
+    for (;;) {
+        uint32_t row32 = 0;
+        if (lane == 0) row32 = atomicAdd(P.next_row, 1u);
+        const int64_t row = __shfl_sync(kFull, row32, 0);
+        if (row >= P.n_rows) break;
+        const int64_t rep = row / per_rep;
+        const int set = (int)((row / P.n_pols) % P.n_sets);
+        const int pol = P.pols[row % P.n_pols];
+        const ConstsDev& cc = P.sets[set];
+        const int64_t n = P.n_req;
+        const int64_t tb = rep * n;
+        const int64_t ob = row * n;
+
+        if (!row_valid(P, tb, lane)) {
+            if (lane == 0) {
+                P.row_status[row] = CTR_EINVAL;
+                P.row_hash[row] = 0;
+            }
+            continue;
+        }
+
+        Decode s;
+        s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.R = 0; s.ohat = 0; s.steps = 0;
+        s.pend_top = kEmpty; s.act_top = kEmpty;
+        s.n_act = 0; s.q = 0; s.pend_n = 0; s.act_n = 0; s.w_head = 0; s.w_n = 0;
+        s.stepping = false;
+        int64_t busy = 0, ring_front = kNever;  // prefill lanes
+        int32_t ring_head = 0, ring_n = 0;
+        int32_t rr_p = 0, rr_d = 0;
+        uint64_t h = 0;
+        int err = CTR_OK;
+
+        for (int64_t base = 0; base < n; base += 32) {
+            const int64_t kl = base + lane;
+            const bool live = kl < n;
+            int64_t my_t = 0;
+            uint32_t my_pc = 0, my_o = 0, my_oh = 0;
+            if (live) {
+                my_t = P.trace.arrival_us[tb + kl];
+                my_pc = (uint32_t)P.trace.prompt_len[tb + kl] | ((uint32_t)P.trace.slo_class[tb + kl] << 24);
+                my_o = (uint32_t)P.trace.true_out[tb + kl];
+                my_oh = (uint32_t)P.trace.pred_out[tb + kl];
+            }
+            uint32_t my_route = 0;
+            const int cnt = (int)(n - base < 32 ? n - base : 32);
+            for (int j = 0; j < cnt; ++j) {
+                const int64_t k = base + j;
+                const int64_t T = __shfl_sync(kFull, my_t, j);
+                const uint32_t pc = __shfl_sync(kFull, my_pc, j);
+                const int64_t pk = pc & 0xFFFFFFu;
+                const int ck = (int)(pc >> 24);
+                const int64_t ok = __shfl_sync(kFull, my_o, j);
+                const int64_t ohk = __shfl_sync(kFull, my_oh, j);
+
+                // 1. advance every instance to the arrival time
+                if (is_dec) {
+                    err = decode_advance(s, T, P, pend, act, wait, tb, ob, h);
+                } else if (is_pre) {
+                    while (ring_n > 0 && ring_front <= T) {
+                        ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
+                        ring_n -= 1;
+                        ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
+                    }
+                }
+                if (__any_sync(kFull, err != CTR_OK)) break;
+
+                // 2. price the candidates and take the argmin of each pool
+                int ip, id;
+                if (pol == CTR_POLICY_ROUND_ROBIN) {
+                    ip = rr_p;
+                    id = rr_d;
+                    rr_p = rr_p + 1 == P.n_pre ? 0 : rr_p + 1;
+                    rr_d = rr_d + 1 == P.n_dec ? 0 : rr_d + 1;
+                } else {
+                    uint64_t cost = kEmpty;
+                    if (is_pre) {
+                        if (pol == CTR_POLICY_LEARNED) {
+                            const int64_t b = busy > T ? busy - T : 0;
+                            const int64_t load = cc.w_b * b + cc.w_s * (cc.tau_pre0 + pk * cc.tau_pre);
+                            cost = (uint64_t)(load * cc.sigma[ck] + cc.w_q * (int64_t)ring_n * 65536);
+                        } else {
+                            cost = (uint64_t)ring_n;
+                        }
+                    } else if (is_dec) {
+                        if (pol == CTR_POLICY_LEARNED) {
+                            const int64_t na = s.n_act;
+                            const int64_t step = P.dec_base + P.dec_seq * na + kv_term(s.kv_res, P);
+                            const uint64_t hi = __umul64hi((uint64_t)s.R, (uint64_t)step);
+                            const uint64_t lo = (uint64_t)s.R * (uint64_t)step;
+                            int64_t b;
+                            if (hi != 0 || lo >= (1ull << 62)) {
+                                b = kBacklogClamp;
+                            } else {
+                                b = (int64_t)(lo / (uint64_t)(na > 1 ? na : 1));
+                                if (b > kBacklogClamp) b = kBacklogClamp;
+                            }
+                            int64_t press = (int64_t)div_recip((uint64_t)(s.kv_res + pk + ohk) << 16,
+                                                               (uint64_t)P.kv_cap, P.kv_cap_recip);
+                            if (press > kPressureClamp) press = kPressureClamp;
+                            const int64_t own = ohk * cc.tau_dec;
+                            const int64_t priced = own + ((((own * press) >> 16) * cc.rho) >> 8);
+                            const int64_t load = cc.w_b * b + cc.w_s * priced;
+                            cost = (uint64_t)(load * cc.sigma[ck] + cc.w_q * (int64_t)s.q * 65536);
+                        } else if (pol == CTR_POLICY_LENGTH_HEURISTIC && ohk >= P.heur_thresh) {
+                            cost = (uint64_t)s.ohat;
+                        } else {
+                            cost = (uint64_t)s.q;
+                        }
+                    }
+                    ip = warp_argmin(is_pre ? cost : kEmpty);
+                    id = warp_argmin(is_dec ? cost : kEmpty) - P.n_pre;
+                }
+
+                // 3. commit: FCFS prefill, KV transfer, queue at the decode instance
+                int64_t ready = 0;
+                if (lane == ip) {
+                    const int64_t start = busy > T ? busy : T;
+                    const int64_t end = start + P.pre_base + P.pre_tok * pk;
+                    ready = end + P.xfer_tok * pk;
+                    if (ready >= kTimeLimit) {
+                        err = CTR_EOVERFLOW;
+                    } else if (ring_n == P.cap_ring) {
+                        err = CTR_EOVERFLOW;
+                    } else {
+                        busy = end;
+                        int pos = ring_head + ring_n;
+                        if (pos >= P.cap_ring) pos -= P.cap_ring;
+                        ring[pos * kWarp] = end;
+                        if (ring_n == 0) ring_front = end;
+                        ring_n += 1;
+                    }
+                }
+                ready = __shfl_sync(kFull, ready, ip);
+                if (lane == P.n_pre + id && ready < kTimeLimit) {
+                    if (s.pend_n == P.cap_pend) {
+                        err = CTR_EOVERFLOW;
+                    } else {
+                        heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
+                        s.q += 1;
+                        s.R += ok;
+                        s.ohat += ohk;
+                    }
+                }
+                if (lane == 0) h += hterm(k, 1, ((uint64_t)ip << 8) | (uint64_t)id);
+                if (lane == j) my_route = ((uint32_t)ip << 8) | (uint32_t)id;
+                if (__any_sync(kFull, err != CTR_OK)) break;
+            }
+            if (__any_sync(kFull, err != CTR_OK)) break;
+            if (live) {
+                if (P.i_pre) P.i_pre[ob + kl] = (uint8_t)(my_route >> 8);
+                if (P.i_dec) P.i_dec[ob + kl] = (uint8_t)(my_route & 0xFF);
+            }
+        }
+        // drain: every remaining event
+        if (!__any_sync(kFull, err != CTR_OK) && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob, h);
+
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off);
+        int status = CTR_OK;
+        if (__any_sync(kFull, err == CTR_ETIMEOUT)) status = CTR_ETIMEOUT;
+        if (__any_sync(kFull, err == CTR_EOVERFLOW)) status = CTR_EOVERFLOW;
+        if (__any_sync(kFull, err == CTR_EINVAL)) status = CTR_EINVAL;
+        if (lane == 0) {
+            P.row_status[row] = status;
+            P.row_hash[row] = status == CTR_OK ? h : 0;
+        }
+    }
+}
+
+}  // namespace
+
+int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr)
+{
+    const int64_t pr = cfg.cap_pending > cfg.cap_prefill_ring ? cfg.cap_pending : cfg.cap_prefill_ring;
+    const int64_t a = pr * 8 * kWarp;
+    const int64_t b = a + (int64_t)cfg.cap_active * 8 * kWarp;
+    const int64_t c = b + (int64_t)cfg.cap_waiting * 4 * kWarp;
+    *off_act = a;
+    *off_wait = b;
+    *cap_pr = (int32_t)pr;
+    return (c + 255) / 256 * 256;
+}
+
+int sim_max_resident_warps(int* warps_per_block, int* blocks)
+{
+    int dev = 0, sms = 0, per_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sim_kernel, kWarpsPerBlock * 32, 0) != cudaSuccess)
+        return 0;
+    *warps_per_block = kWarpsPerBlock;
+    *blocks = sms * per_sm;
+    return sms * per_sm * kWarpsPerBlock;
+}
+
+cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
+{
+    (void)warps_per_block;
+    sim_kernel<<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace ctr

@@ -1,0 +1,81 @@
+"""The C ABI library (no GPU needed): it loads, exports every function that
+include/ctr.h declares, its ctypes binding lays structs out exactly as the
+header does, and the product path refuses to run without CUDA."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from conftest import ROOT
+
+HEADER = os.path.join(ROOT, "include", "ctr.h")
+
+
+@pytest.fixture(scope="module")
+def libctr():
+    from paper_2609_16206_gb300 import build
+    path = build.build()
+    return ctypes.CDLL(path)
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b(ctr_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_exports_every_declared_function(libctr):
+    names = declared_functions()
+    assert {"ctr_gen_trace", "ctr_score_batch", "ctr_simulate", "ctr_goodput"} <= set(names)
+    for name in names:
+        assert hasattr(libctr, name), name
+
+
+def test_static_entry_points_run_without_gpu(libctr):
+    libctr.ctr_strerror.restype = ctypes.c_char_p
+    assert libctr.ctr_strerror(-3).decode().startswith("a fixed-capacity")
+    assert libctr.ctr_abi_version() == 1
+
+
+def test_struct_layout_matches_header(tmp_path):
+    from paper_2609_16206_gb300 import ctr
+    structs = {"ctr_requests": ctr.CtrRequests, "ctr_trace_cfg": ctr.CtrTraceCfg, "ctr_sim_cfg": ctr.CtrSimCfg,
+               "ctr_cost_consts": ctr.CtrCostConsts}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HEADER}"', "int main(void){"]
+    for cname, py in structs.items():
+        lines.append(f'printf("{cname} sizeof %zu\\n", sizeof({cname}));')
+        for field, _ in py._fields_:
+            lines.append(f'printf("{cname} {field} %zu\\n", offsetof({cname}, {field}));')
+    lines.append("return 0;}")
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c11", "-o", str(exe), str(src)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split("\n")
+    got = {tuple(l.split()[:2]): int(l.split()[2]) for l in out if l.strip()}
+    for cname, py in structs.items():
+        assert got[(cname, "sizeof")] == ctypes.sizeof(py), cname
+        for field, _ in py._fields_:
+            assert got[(cname, field)] == getattr(py, field).offset, (cname, field)
+
+
+def test_product_path_fails_loudly_without_cuda():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    from paper_2609_16206_gb300 import ctr
+    from paper_2609_16206_gb300 import workloads as W
+    with pytest.raises(Exception):
+        tr = ctr.empty_requests(1, 10, "cpu")
+        ctr.ctr_gen_trace(W.TraceCfg(), 1, 0, 10, tr)
+
+
+def test_workspace_query_without_gpu_is_zero():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    from paper_2609_16206_gb300 import ctr
+    from paper_2609_16206_gb300 import workloads as W
+    assert ctr.ctr_workspace_bytes(0, W.SimCfg(), 4, 100) == 0

@@ -1,0 +1,133 @@
+"""Parity: the fp32 GPU scorer against the fp64 brute-force oracle -- relative
+error <= 1e-6 per cost, identical argmin except where the oracle's top-two gap
+is below 1e-5 relative (there the GPU's pick must itself be within 1e-5 of
+the minimum)."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from conftest import GOLDEN
+from gpuutil import need_gpu
+from paper_2609_16206_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+REL_COST = 1e-6
+REL_GAP = 1e-5
+
+
+def _run(ctr, p, oh, cls, Q, A, kap, consts, offset=0):
+    dev = "cuda"
+
+    def t(a, dt):  # optional element offset to break 16-byte alignment
+        buf = torch.zeros(a.size + offset, dtype=dt, device=dev)
+        buf[offset:] = torch.from_numpy(np.ascontiguousarray(a))
+        return buf[offset:]
+    n = p.size
+    am = torch.full((n + offset,), -9, dtype=torch.int32, device=dev)[offset:]
+    cost = torch.full((n + offset,), -9.0, dtype=torch.float32, device=dev)[offset:]
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    ctr.ctr_score_batch(t(p, torch.float32), t(oh, torch.float32), t(cls, torch.uint8), t(Q, torch.float32),
+                        t(A, torch.float32), t(kap, torch.float32), consts, am, cost, status=status)
+    torch.cuda.synchronize()
+    assert int(status[0]) == 0
+    return am.cpu().numpy(), cost.cpu().numpy()
+
+
+def _check(orc, p, oh, cls, Q, A, kap, consts, am, cost):
+    ref_am, best, second = orc.score_batch(p, oh, cls, Q, A, kap, consts)
+    bad_cls = cls >= 4
+    assert np.all(am[bad_cls] == -1) and np.all(np.isnan(cost[bad_cls]))
+    ok = ~bad_cls
+    gap = (second - best) / best
+    strict = ok & (gap >= REL_GAP)
+    assert np.array_equal(am[strict], ref_am[strict]), np.flatnonzero(am[strict] != ref_am[strict])[:5]
+    idx = np.flatnonzero(ok)
+    if idx.size == 0:
+        return 0
+    chosen = orc.score_pairs(p, oh, cls, idx, am[idx], Q, A, kap, consts)
+    assert np.all(chosen <= best[idx] * (1 + REL_GAP) + 1e-30)
+    rel = np.abs(cost[idx].astype(np.float64) - chosen) / np.maximum(chosen, 1e-30)
+    assert rel.max() <= REL_COST, rel.max()
+    return int((ok & ~strict).sum())
+
+
+def test_standalone_batch_full_size(orc):
+    """2^20 requests x 64 instances, the standalone scoring workload."""
+    ctr = need_gpu()
+    p, oh, cls = W.score_requests(1 << 20, seed=0)
+    Q, A, kap = W.score_state(64, seed=1)
+    am, cost = _run(ctr, p, oh, cls, Q, A, kap, W.SCORE_CONSTS)
+    near = _check(orc, p, oh, cls, Q, A, kap, W.SCORE_CONSTS, am, cost)
+    assert near < 1000
+
+
+@pytest.mark.parametrize("n", [0, 1, 3, 5, 4097, 100_003])
+@pytest.mark.parametrize("offset", [0, 1])
+def test_ragged_and_misaligned(orc, n, offset):
+    ctr = need_gpu()
+    p, oh, cls = W.score_requests(n, seed=n + 3)
+    Q, A, kap = W.score_state(64, seed=4)
+    am, cost = _run(ctr, p, oh, cls, Q, A, kap, W.SCORE_CONSTS, offset=offset)
+    _check(orc, p, oh, cls, Q, A, kap, W.SCORE_CONSTS, am, cost)
+
+
+@pytest.mark.parametrize("n_inst", [1, 2, 7, 63, 64, 65, 256])
+def test_instance_counts(orc, n_inst):
+    ctr = need_gpu()
+    p, oh, cls = W.score_requests(20_000, seed=n_inst)
+    Q, A, kap = W.score_state(n_inst, seed=n_inst + 1)
+    am, cost = _run(ctr, p, oh, cls, Q, A, kap, W.SCORE_CONSTS)
+    _check(orc, p, oh, cls, Q, A, kap, W.SCORE_CONSTS, am, cost)
+
+
+def test_degenerate_states(orc):
+    ctr = need_gpu()
+    p, oh, cls = W.score_requests(30_000, seed=77)
+    cls = cls.copy()
+    cls[::97] = 4
+    cls[::101] = 255
+    Q, A, kap = W.score_state(16, seed=78)
+    cases = [
+        (np.repeat(Q[:4], 4), np.repeat(A[:4], 4), np.repeat(kap[:4], 4)),   # duplicated instances
+        (Q, A, np.zeros_like(kap)),                                            # no KV pressure
+        (np.zeros_like(Q), np.zeros_like(A), kap),                             # idle pool
+        (np.full_like(Q, 5.0), np.full_like(A, 3.0), np.full_like(kap, 0.5)),  # all equal
+    ]
+    for Qc, Ac, kc in cases:
+        am, cost = _run(ctr, p, oh, cls, Qc, Ac, kc, W.SCORE_CONSTS)
+        _check(orc, p, oh, cls, Qc, Ac, kc, W.SCORE_CONSTS, am, cost)
+    zero_rho = W.SCORE_CONSTS.copy()
+    zero_rho[3] = 0.0
+    am, cost = _run(ctr, p, oh, cls, Q, A, kap, zero_rho)
+    _check(orc, p, oh, cls, Q, A, kap, zero_rho, am, cost)
+
+
+def test_hand_computed_exact(orc):
+    ctr = need_gpu()
+    with open(os.path.join(GOLDEN, "score_hand.json")) as f:
+        h = json.load(f)
+    r, s, e = h["requests"], h["state"], h["expect"]
+    f32 = lambda x: np.array(x, np.float32)
+    am, cost = _run(ctr, f32(r["p"]), f32(r["oh"]), np.array(r["cls"], np.uint8), f32(s["Q"]), f32(s["A"]),
+                    f32(s["kappa"]), np.array(h["consts"], np.float32))
+    assert am[3] == -1 and np.isnan(cost[3])
+    # requests 0..2 tie between instances 2 and 3: either is a valid argmin, the cost is exact
+    assert set(am[:3].tolist()) <= {2, 3}
+    assert cost[:3].tolist() == e["best"][:3]
+
+
+def test_invalid_arguments():
+    ctr = need_gpu()
+    x = torch.zeros(8, device="cuda")
+    c = torch.zeros(8, dtype=torch.uint8, device="cuda")
+    am = torch.zeros(8, dtype=torch.int32, device="cuda")
+    bad = W.SCORE_CONSTS.copy()
+    bad[0] = -1.0
+    with pytest.raises(ctr.CtrError):
+        ctr.ctr_score_batch(x, x, c, x, x, x, bad, am, x)
+    big = torch.zeros(257, device="cuda")
+    with pytest.raises(ctr.CtrError):
+        ctr.ctr_score_batch(x, x, c, big, big, big, W.SCORE_CONSTS, am, x)

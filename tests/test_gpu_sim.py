@@ -1,0 +1,204 @@
+"""Parity: the GPU replica simulator matches the CPU oracle bit for bit --
+every routing decision, first-token and completion time, and the row hash --
+on hand-made traces, generated workloads, several constant sets, the widest
+pool, ragged and empty inputs, and the error paths."""
+import numpy as np
+import pytest
+import torch
+
+import simutil as U
+from gpuutil import gen, host_trace, need_gpu, simulate, to_dev
+from paper_2609_16206_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _check_rows(orc, sc, sets, pols, tr_host_rows, res, n_req, full=True):
+    row = 0
+    for r, trh in enumerate(tr_host_rows):
+        for cc in sets:
+            for pol in pols:
+                o = orc.simulate(sc, cc, pol, trh)
+                assert res["status"][row] == o["status"], (row, res["status"][row], o["status"])
+                if o["status"] == 0:
+                    assert int(res["hash"][row]) == o["hash"], row
+                    if full:
+                        for key in ("t_first_us", "t_done_us", "i_pre", "i_dec"):
+                            if key in res:
+                                got, want = res[key][row], o[key]
+                                assert np.array_equal(got, want), (key, row, np.flatnonzero(got != want)[:5])
+                row += 1
+
+
+@pytest.mark.parametrize("case", U.worked_traces(), ids=lambda c: c["name"])
+def test_worked_traces(orc, case):
+    ctr = need_gpu()
+    sc = U.sim_from(case["sim"])
+    trh = U.trace_from(case["requests"])
+    sets = [U.consts_from(case["consts"])]
+    res = simulate(ctr, sc, sets, list(W.ALL_POLICIES), to_dev(trh), 1, trh["arrival_us"].size)
+    _check_rows(orc, sc, sets, list(W.ALL_POLICIES), [trh], res, trh["arrival_us"].size)
+    # and the hand-derived values themselves
+    j = list(W.ALL_POLICIES).index(case["policy"])
+    for key in ("t_first_us", "t_done_us", "i_pre", "i_dec"):
+        if key in case["expect"]:
+            assert res[key][j].tolist() == case["expect"][key]
+
+
+def test_single_replica_all_policies(orc):
+    ctr = need_gpu()
+    wl = W.single_replica()
+    tr = gen(ctr, wl.trace, 1, wl.n_req)
+    res = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, 1, wl.n_req)
+    _check_rows(orc, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), [host_trace(tr, 0)], res, wl.n_req)
+
+
+def test_bursty_replicas_all_policies(orc):
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    R, N = 20, 3000
+    tr = gen(ctr, wl.trace, R, N)
+    res = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, R, N)
+    _check_rows(orc, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), [host_trace(tr, r) for r in range(R)], res, N)
+
+
+def test_mispriced_constant_sets(orc):
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    sets = W.mispriced_sets()[::9]
+    R, N = 3, 1500
+    tr = gen(ctr, wl.trace, R, N)
+    res = simulate(ctr, wl.sim, sets, [W.POLICY_LEARNED, W.POLICY_JSQ], tr, R, N)
+    _check_rows(orc, wl.sim, sets, [W.POLICY_LEARNED, W.POLICY_JSQ], [host_trace(tr, r) for r in range(R)], res, N)
+
+
+def test_large_pool_overload(orc):
+    """4P+28D (all 32 lanes) at prefill overload: deep queues, three classes."""
+    ctr = need_gpu()
+    wl = W.large_pool(rate_mreq=34_000)
+    R, N = 2, 4000
+    tr = gen(ctr, wl.trace, R, N)
+    cc = wl.consts[0]
+    res = simulate(ctr, wl.sim, [cc], list(W.ALL_POLICIES), tr, R, N)
+    _check_rows(orc, wl.sim, [cc], list(W.ALL_POLICIES), [host_trace(tr, r) for r in range(R)], res, N)
+
+
+@pytest.mark.parametrize("n_pre,n_dec", [(1, 1), (31, 1), (1, 31), (3, 5)])
+def test_pool_shapes(orc, n_pre, n_dec):
+    ctr = need_gpu()
+    sc = W.SimCfg(n_prefill=n_pre, n_decode=n_dec)
+    tc = W.TraceCfg(rate_mreq=(3000, 3000), seed=n_pre * 100 + n_dec)
+    N = 700
+    tr = gen(ctr, tc, 2, N)
+    res = simulate(ctr, sc, [W.CALIBRATED], list(W.ALL_POLICIES), tr, 2, N)
+    _check_rows(orc, sc, [W.CALIBRATED], list(W.ALL_POLICIES), [host_trace(tr, r) for r in range(2)], res, N)
+
+
+@pytest.mark.parametrize("N", [0, 1, 31, 33, 65])
+def test_ragged_and_empty(orc, N):
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    tr = gen(ctr, wl.trace, 2, N)
+    res = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, 2, N)
+    _check_rows(orc, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), [host_trace(tr, r) for r in range(2)], res, N)
+
+
+def test_small_workspace_same_results(orc):
+    """A workspace with room for only two warp slots runs the rows in turn."""
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    R, N = 6, 800
+    tr = gen(ctr, wl.trace, R, N)
+    full = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, R, N)
+    slot = ctr.ctr_workspace_bytes(0, wl.sim, 1, N) - 256
+    small = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, R, N, ws_bytes=256 + 2 * slot)
+    for key in full:
+        assert np.array_equal(full[key], small[key]), key
+
+
+def test_routes_optional(orc):
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    tr = gen(ctr, wl.trace, 2, 500)
+    a = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, 2, 500, routes=False)
+    b = simulate(ctr, wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, 2, 500)
+    assert np.array_equal(a["hash"], b["hash"]) and np.array_equal(a["t_done_us"], b["t_done_us"])
+
+
+def test_capacity_overflow_matches_oracle(orc):
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    N = 2000
+    tr = gen(ctr, wl.trace, 1, N)
+    trh = host_trace(tr, 0)
+    st = orc.simulate(wl.sim, W.CALIBRATED, W.POLICY_LEARNED, trh)["stats"]
+    caps = dict(cap_pending=st["max_pending"], cap_waiting=st["max_waiting"], cap_active=st["max_active"],
+                cap_prefill_ring=st["max_prefill"])
+    ok = simulate(ctr, wl.sim.replace(**caps), [W.CALIBRATED], [W.POLICY_LEARNED], tr, 1, N)
+    assert ok["status"][0] == 0
+    for name in caps:
+        if caps[name] <= 1:
+            continue
+        tight = dict(caps)
+        tight[name] -= 1
+        bad = simulate(ctr, wl.sim.replace(**tight), [W.CALIBRATED], [W.POLICY_LEARNED], tr, 1, N)
+        assert bad["status"][0] == ctr.CTR_EOVERFLOW, name
+
+
+def test_step_budget_and_invalid_rows(orc):
+    ctr = need_gpu()
+    wl = W.single_replica()
+    N = 300
+    trh = orc.gen_trace(wl.trace, N)
+    res = simulate(ctr, wl.sim.replace(max_steps_per_instance=50), [W.CALIBRATED], [W.POLICY_RR], to_dev(trh), 1, N)
+    assert res["status"][0] == ctr.CTR_ETIMEOUT
+    bad = dict(trh)
+    bad["true_out"] = trh["true_out"].copy()
+    bad["true_out"][7] = 0
+    rows = {k: np.stack([trh[k], bad[k]]) for k in trh}
+    res = simulate(ctr, wl.sim, [W.CALIBRATED], [W.POLICY_LEARNED], to_dev(rows), 2, N)
+    assert res["status"].tolist() == [0, ctr.CTR_EINVAL]
+    assert int(res["hash"][0]) == orc.simulate(wl.sim, W.CALIBRATED, 0, trh)["hash"]
+    un = dict(trh)
+    un["arrival_us"] = trh["arrival_us"].copy()
+    un["arrival_us"][40] = un["arrival_us"][39] - 1
+    assert simulate(ctr, wl.sim, [W.CALIBRATED], [0], to_dev(un), 1, N)["status"][0] == ctr.CTR_EINVAL
+
+
+def test_host_validation_rejects(orc):
+    ctr = need_gpu()
+    wl = W.single_replica()
+    tr = gen(ctr, wl.trace, 1, 50)
+    for sc, sets, pols in ((wl.sim.replace(n_prefill=0), [W.CALIBRATED], [0]),
+                           (wl.sim.replace(n_prefill=20, n_decode=13), [W.CALIBRATED], [0]),
+                           (wl.sim, [W.CALIBRATED.replace(w_b_q8=1024)], [0]),
+                           (wl.sim, [W.CALIBRATED], [4]),
+                           (wl.sim, [W.CALIBRATED], []),
+                           (wl.sim.replace(cap_active=0), [W.CALIBRATED], [0])):
+        with pytest.raises(Exception):
+            simulate(ctr, sc, sets, pols, tr, 1, 50)
+
+
+def test_full_size_sweep_sampled(orc):
+    """The benchmarked configuration in the benchmark's launch shape: 4,096 bursty
+    replicas x 20,000 requests x 4 policies in one launch; sampled rows against
+    the oracle by hash (every row's status must be OK)."""
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    R, N = wl.n_replicas, wl.n_req
+    tr = gen(ctr, wl.trace, R, N)
+    rows = R * 4
+    tf = torch.empty((rows, N), dtype=torch.int64, device="cuda")
+    td = torch.empty_like(tf)
+    h = torch.empty(rows, dtype=torch.int64, device="cuda")
+    st = torch.empty(rows, dtype=torch.int32, device="cuda")
+    ws = ctr.simulate_workspace(wl.sim, rows, N, "cuda")
+    ctr.ctr_simulate(wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, R, N, tf, td, h, st, ws)
+    torch.cuda.synchronize()
+    assert int((st != 0).sum()) == 0
+    hh = h.cpu().numpy().astype(np.uint64)
+    for r in (0, 1, 2, 2048, 4095):
+        trh = host_trace(tr, r)
+        for j, pol in enumerate(W.ALL_POLICIES):
+            o = orc.simulate(wl.sim, W.CALIBRATED, pol, trh)
+            assert o["status"] == 0 and int(hh[r * 4 + j]) == o["hash"], (r, pol)
