@@ -8,7 +8,8 @@
  *     the host before any launch; a rejected call launches nothing.
  *   - Arrays are DEVICE pointers owned by the caller unless marked "host".
  *     The library allocates nothing and keeps no state between calls, so calls
- *     on different streams are independent and thread-safe.
+ *     on different streams are independent and thread-safe (the one exception,
+ *     ctr_simulate_noalloc, documents its shared scratch array).
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Work is enqueued asynchronously; nothing synchronises unless
  *     stated.  Launch failures are reported as CTR_ECUDA.
@@ -172,6 +173,28 @@ int ctr_simulate(const ctr_sim_cfg* cfg /* host */, const ctr_cost_consts* const
                  const int32_t* policy_ids /* host */, int32_t n_policies, ctr_requests trace, int32_t n_replicas,
                  int64_t n_req, uint8_t* i_pre, uint8_t* i_dec, int64_t* t_first_us, int64_t* t_done_us,
                  uint64_t* row_hash, int32_t* row_status, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ctr_simulate_noalloc -- ctr_simulate for callers that cannot allocate
+ * device memory (the paper has no counterpart: this is a deployment aid).
+ * Some callers run where a device allocation is not theirs to make -- a
+ * plugin inside a serving process whose memory pool owns the GPU, code
+ * between someone else's stream-capture calls, a loop that must never reach
+ * the driver's allocator.  This entry point takes the simulator's scratch
+ * from a fixed array of CTR_NOALLOC_SCRATCH_BYTES that the library keeps on
+ * every GPU it is loaded on until the process exits; the caller still owns
+ * and passes the trace and every output, exactly as for ctr_simulate, and the
+ * results are identical.  The first call on a device looks the array up (once
+ * per device); make it before any stream capture.  All calls share the array:
+ * calls that overlap on the GPU (two streams, two threads) race and must be
+ * serialised.  A configuration whose per-warp structures (the cap_* fields)
+ * do not fit the array returns CTR_EINVAL; otherwise fewer rows run at once
+ * than with a full workspace.  Allocates nothing. */
+#define CTR_NOALLOC_SCRATCH_BYTES ((size_t)64 << 20)
+int ctr_simulate_noalloc(const ctr_sim_cfg* cfg /* host */, const ctr_cost_consts* consts /* host */,
+                         int32_t n_const_sets, const int32_t* policy_ids /* host */, int32_t n_policies,
+                         ctr_requests trace, int32_t n_replicas, int64_t n_req, uint8_t* i_pre, uint8_t* i_dec,
+                         int64_t* t_first_us, int64_t* t_done_us, uint64_t* row_hash, int32_t* row_status,
+                         void* stream);
 
 /* ctr_goodput -- SLO goodput inputs per row (sec. IV-B targets, Table 2
  * columns): met_count[row] = #{k : TTFT <= TTFT_c and (o == 1 or

@@ -18,7 +18,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OBJ = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libctr.so")
-SOURCES = ["api.cu", "trace.cu", "sim.cu", "score.cu", "goodput.cu"]
+SOURCES = ["api.cu", "trace.cu", "sim.cu", "score.cu", "goodput.cu", "noalloc.cu"]
 HEADERS = [os.path.join(CSRC, "ctr_internal.cuh"), os.path.join(ROOT, "include", "ctr.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",

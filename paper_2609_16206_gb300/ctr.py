@@ -92,6 +92,9 @@ def lib():
             L.ctr_simulate.argtypes = [C.POINTER(CtrSimCfg), C.POINTER(CtrCostConsts), i32, C.POINTER(i32), i32,
                                        CtrRequests, i32, i64, vp, vp, vp, vp, vp, vp, vp, C.c_size_t, vp]
             L.ctr_simulate.restype = C.c_int
+            L.ctr_simulate_noalloc.argtypes = [C.POINTER(CtrSimCfg), C.POINTER(CtrCostConsts), i32, C.POINTER(i32),
+                                               i32, CtrRequests, i32, i64, vp, vp, vp, vp, vp, vp, vp]
+            L.ctr_simulate_noalloc.restype = C.c_int
             L.ctr_goodput.argtypes = [C.POINTER(CtrSimCfg), CtrRequests, i32, i32, i64, vp, vp, vp, vp, vp]
             L.ctr_goodput.restype = C.c_int
             L.ctr_strerror.argtypes = [C.c_int]
@@ -232,6 +235,19 @@ def ctr_simulate(sim_cfg, const_sets, policies, trace: dict, n_replicas: int, n_
         C.byref(cfg), sets, len(sets), pols, len(policies), requests_struct(trace), int(n_replicas), int(n_req),
         _ptr(i_pre), _ptr(i_dec), _ptr(t_first_us), _ptr(t_done_us), _ptr(row_hash), _ptr(row_status),
         _ptr(workspace), int(workspace.numel() * workspace.element_size()), _stream(stream)))
+
+
+def ctr_simulate_noalloc(sim_cfg, const_sets, policies, trace: dict, n_replicas: int, n_req: int, t_first_us,
+                         t_done_us, row_hash, row_status, i_pre=None, i_dec=None, stream=None):
+    """ctr_simulate without a workspace: the library's fixed scratch array is
+    used instead, for callers that cannot allocate device memory."""
+    cfg = sim_cfg_struct(sim_cfg)
+    sets = consts_array(list(const_sets))
+    pols = (C.c_int32 * len(policies))(*[int(p) for p in policies])
+    _check("ctr_simulate_noalloc", lib().ctr_simulate_noalloc(
+        C.byref(cfg), sets, len(sets), pols, len(policies), requests_struct(trace), int(n_replicas), int(n_req),
+        _ptr(i_pre), _ptr(i_dec), _ptr(t_first_us), _ptr(t_done_us), _ptr(row_hash), _ptr(row_status),
+        _stream(stream)))
 
 
 def ctr_goodput(sim_cfg, trace: dict, n_replicas: int, rows_per_replica: int, n_req: int, t_first_us, t_done_us,
