@@ -176,7 +176,7 @@ def run_ours(args, rank, world, local_rank):
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
     stream = torch.cuda.current_stream()
-    wl = W.replica_sweep()
+    wl = W.replica_sweep(n_replicas=args.replicas or 4096, n_req=args.requests or 20_000)
     R, N = wl.n_replicas, wl.n_req
     pols = list(W.ALL_POLICIES)
     rows = R * len(pols)
@@ -287,6 +287,8 @@ def run_ours(args, rank, world, local_rank):
         out_host["cost"].copy_(scost, non_blocking=True)
         torch.cuda.synchronize()
 
+    if args.no_e2e:
+        e2e_step = lambda: None  # noqa: E731
     e2e_step()
     e2e_steps = max(1, min(args.steps, 3))
     if world > 1:
@@ -298,7 +300,7 @@ def run_ours(args, rank, world, local_rank):
     e2e_t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
     if world > 1:
         torch.distributed.all_reduce(e2e_t, op=torch.distributed.ReduceOp.MAX)
-    e2e_value = routed_per_step / float(e2e_t.item())
+    e2e_value = None if args.no_e2e else routed_per_step / float(e2e_t.item())
 
     if rank != 0:
         return 0
@@ -361,6 +363,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end pass")
+    ap.add_argument("--replicas", type=int, default=None,
+                    help="replicas per GPU (profiling a smaller case; default: the benchmarked 4,096)")
+    ap.add_argument("--requests", type=int, default=None, help="requests per replica (default 20,000)")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
