@@ -254,7 +254,9 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     if (workspace_bytes < 256 + (size_t)p.slot_bytes) return CTR_EINVAL;
     int64_t slots = (int64_t)((workspace_bytes - 256) / (size_t)p.slot_bytes);
     if (slots > resident) slots = resident;
-    if (slots > n_rows) slots = n_rows;
+    const int64_t rows_per_warp = 32 / sim_group_width(cfg->n_prefill + cfg->n_decode);
+    const int64_t warps_needed = (n_rows + rows_per_warp - 1) / rows_per_warp;
+    if (slots > warps_needed) slots = warps_needed;
     p.n_slots = (int32_t)slots;
     p.ws = static_cast<unsigned char*>(workspace) + 256;
     p.next_row = static_cast<uint32_t*>(workspace);

@@ -71,6 +71,7 @@ struct SimParams {
 };
 int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr);
 int sim_max_resident_warps(int* warps_per_block, int* blocks);
+int sim_group_width(int n_instances);  // lanes per simulated row; 32 / width rows share a warp
 cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream);
 
 // ---------------------------------------------------------------- goodput

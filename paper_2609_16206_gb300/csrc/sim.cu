@@ -230,9 +230,42 @@ __device__ __forceinline__ bool row_valid(const SimParams& P, int64_t tb, int la
     return true;
 }
 
+// argmin of 64-bit values within aligned groups of G lanes (ties -> lowest lane),
+// returned as the lane index inside the group
+template <int G>
+__device__ __forceinline__ int group_argmin(uint64_t v, int gl)
+{
+    if constexpr (G == 32) {
+        return warp_argmin(v);
+    } else {
+        int idx = gl;
+#pragma unroll
+        for (int off = G / 2; off > 0; off >>= 1) {
+            const uint64_t ov = __shfl_xor_sync(kFull, v, off, G);
+            const int oi = __shfl_xor_sync(kFull, idx, off, G);
+            if (ov < v || (ov == v && oi < idx)) {
+                v = ov;
+                idx = oi;
+            }
+        }
+        return idx;
+    }
+}
+
+// One warp carries 32 / G rows side by side: lanes [g*G, g*G + G) simulate
+// row base_row + g, lane g*G + i being instance i of that row.  All rows of a
+// workload have the same number of requests, so the groups walk their
+// arrivals in lockstep (request k of every row at once, each at its own time);
+// the per-lane event loops, the per-group argmins and the commits are
+// independent across groups.
+template <int G>
 __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_constant__ SimParams P)
 {
+    constexpr int kRowsPerWarp = 32 / G;
     const int lane = threadIdx.x & 31;
+    const int grp = lane / G;
+    const int gl = lane % G;
+    const uint32_t gmask = G == 32 ? kFull : (((1u << G) - 1u) << (grp * G));
     const int64_t slot = (int64_t)blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
     if (slot >= P.n_slots) return;
     unsigned char* sb = P.ws + slot * P.slot_bytes;
@@ -241,30 +274,34 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_c
     uint64_t* act = reinterpret_cast<uint64_t*>(sb + P.off_act) + lane;
     uint32_t* wait = reinterpret_cast<uint32_t*>(sb + P.off_wait) + lane;
 
-    const bool is_pre = lane < P.n_pre;
-    const bool is_dec = lane >= P.n_pre && lane < P.n_pre + P.n_dec;
+    const bool is_pre = gl < P.n_pre;
+    const bool is_dec = gl >= P.n_pre && gl < P.n_pre + P.n_dec;
     const int64_t per_rep = (int64_t)P.n_sets * P.n_pols;
+    const int64_t n = P.n_req;
 
     for (;;) {
-        uint32_t row32 = 0;
-        if (lane == 0) row32 = atomicAdd(P.next_row, 1u);
-        const int64_t row = __shfl_sync(kFull, row32, 0);
-        if (row >= P.n_rows) break;
-        const int64_t rep = row / per_rep;
-        const int set = (int)((row / P.n_pols) % P.n_sets);
-        const int pol = P.pols[row % P.n_pols];
+        uint32_t base32 = 0;
+        if (lane == 0) base32 = atomicAdd(P.next_row, (uint32_t)kRowsPerWarp);
+        const int64_t base_row = __shfl_sync(kFull, base32, 0);
+        if (base_row >= P.n_rows) break;
+        const int64_t row = base_row + grp;
+        const bool has_row = row < P.n_rows;
+        const int64_t rep = has_row ? row / per_rep : 0;
+        const int set = has_row ? (int)((row / P.n_pols) % P.n_sets) : 0;
+        const int pol = has_row ? P.pols[row % P.n_pols] : CTR_POLICY_ROUND_ROBIN;
         const ConstsDev& cc = P.sets[set];
-        const int64_t n = P.n_req;
         const int64_t tb = rep * n;
         const int64_t ob = row * n;
 
-        if (!row_valid(P, tb, lane)) {
-            if (lane == 0) {
-                P.row_status[row] = CTR_EINVAL;
-                P.row_hash[row] = 0;
-            }
-            continue;
+        // per-request bounds, one row at a time with the whole warp
+        bool valid = false;
+        for (int g = 0; g < kRowsPerWarp; ++g) {
+            const int64_t r = base_row + g;
+            if (r >= P.n_rows) break;
+            const bool ok = row_valid(P, (r / per_rep) * n, lane);
+            if (g == grp) valid = ok;
         }
+        bool live = has_row && valid;
 
         Decode s;
         s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.R = 0; s.ohat = 0; s.steps = 0;
@@ -277,49 +314,46 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_c
         uint64_t h = 0;
         int err = CTR_OK;
 
-        for (int64_t base = 0; base < n; base += 32) {
-            const int64_t kl = base + lane;
-            const bool live = kl < n;
+        for (int64_t base = 0; base < n; base += G) {
+            if (!__any_sync(kFull, live)) break;
+            const int64_t kl = base + gl;
+            const bool mine = live && kl < n;
             int64_t my_t = 0;
             uint32_t my_pc = 0, my_o = 0, my_oh = 0;
-            if (live) {
+            if (mine) {
                 my_t = P.trace.arrival_us[tb + kl];
                 my_pc = (uint32_t)P.trace.prompt_len[tb + kl] | ((uint32_t)P.trace.slo_class[tb + kl] << 24);
                 my_o = (uint32_t)P.trace.true_out[tb + kl];
                 my_oh = (uint32_t)P.trace.pred_out[tb + kl];
             }
             uint32_t my_route = 0;
-            const int cnt = (int)(n - base < 32 ? n - base : 32);
+            const int cnt = (int)(n - base < G ? n - base : G);
             for (int j = 0; j < cnt; ++j) {
                 const int64_t k = base + j;
-                const int64_t T = __shfl_sync(kFull, my_t, j);
-                const uint32_t pc = __shfl_sync(kFull, my_pc, j);
+                const int64_t T = __shfl_sync(kFull, my_t, j, G);
+                const uint32_t pc = __shfl_sync(kFull, my_pc, j, G);
                 const int64_t pk = pc & 0xFFFFFFu;
                 const int ck = (int)(pc >> 24);
-                const int64_t ok = __shfl_sync(kFull, my_o, j);
-                const int64_t ohk = __shfl_sync(kFull, my_oh, j);
+                const int64_t ok = __shfl_sync(kFull, my_o, j, G);
+                const int64_t ohk = __shfl_sync(kFull, my_oh, j, G);
 
                 // 1. advance every instance to the arrival time
-                if (is_dec) {
-                    err = decode_advance(s, T, P, pend, act, wait, tb, ob, h);
-                } else if (is_pre) {
-                    while (ring_n > 0 && ring_front <= T) {
-                        ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
-                        ring_n -= 1;
-                        ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
+                if (live) {
+                    if (is_dec) {
+                        err = decode_advance(s, T, P, pend, act, wait, tb, ob, h);
+                    } else if (is_pre) {
+                        while (ring_n > 0 && ring_front <= T) {
+                            ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
+                            ring_n -= 1;
+                            ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
+                        }
                     }
                 }
-                if (__any_sync(kFull, err != CTR_OK)) break;
+                if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
 
                 // 2. price the candidates and take the argmin of each pool
-                int ip, id;
-                if (pol == CTR_POLICY_ROUND_ROBIN) {
-                    ip = rr_p;
-                    id = rr_d;
-                    rr_p = rr_p + 1 == P.n_pre ? 0 : rr_p + 1;
-                    rr_d = rr_d + 1 == P.n_dec ? 0 : rr_d + 1;
-                } else {
-                    uint64_t cost = kEmpty;
+                uint64_t cost = kEmpty;
+                if (live && pol != CTR_POLICY_ROUND_ROBIN) {
                     if (is_pre) {
                         if (pol == CTR_POLICY_LEARNED) {
                             const int64_t b = busy > T ? busy - T : 0;
@@ -354,13 +388,23 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_c
                             cost = (uint64_t)s.q;
                         }
                     }
-                    ip = warp_argmin(is_pre ? cost : kEmpty);
-                    id = warp_argmin(is_dec ? cost : kEmpty) - P.n_pre;
                 }
+                const int amin_p = group_argmin<G>(is_pre ? cost : kEmpty, gl);
+                const int amin_d = group_argmin<G>(is_dec ? cost : kEmpty, gl);
+                int ip, id;
+                if (pol == CTR_POLICY_ROUND_ROBIN) {
+                    ip = rr_p;
+                    id = rr_d;
+                } else {
+                    ip = amin_p;
+                    id = amin_d - P.n_pre;
+                }
+                rr_p = rr_p + 1 == P.n_pre ? 0 : rr_p + 1;
+                rr_d = rr_d + 1 == P.n_dec ? 0 : rr_d + 1;
 
                 // 3. commit: FCFS prefill, KV transfer, queue at the decode instance
                 int64_t ready = 0;
-                if (lane == ip) {
+                if (live && gl == ip) {
                     const int64_t start = busy > T ? busy : T;
                     const int64_t end = start + P.pre_base + P.pre_tok * pk;
                     ready = end + P.xfer_tok * pk;
@@ -377,8 +421,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_c
                         ring_n += 1;
                     }
                 }
-                ready = __shfl_sync(kFull, ready, ip);
-                if (lane == P.n_pre + id && ready < kTimeLimit) {
+                ready = __shfl_sync(kFull, ready, ip, G);
+                if (live && gl == P.n_pre + id && ready < kTimeLimit) {
                     if (s.pend_n == P.cap_pend) {
                         err = CTR_EOVERFLOW;
                     } else {
@@ -388,26 +432,25 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_c
                         s.ohat += ohk;
                     }
                 }
-                if (lane == 0) h += hterm(k, 1, ((uint64_t)ip << 8) | (uint64_t)id);
-                if (lane == j) my_route = ((uint32_t)ip << 8) | (uint32_t)id;
-                if (__any_sync(kFull, err != CTR_OK)) break;
+                if (live && gl == 0) h += hterm(k, 1, ((uint64_t)ip << 8) | (uint64_t)id);
+                if (gl == j) my_route = ((uint32_t)ip << 8) | (uint32_t)id;
+                if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
             }
-            if (__any_sync(kFull, err != CTR_OK)) break;
-            if (live) {
+            if (mine && live) {
                 if (P.i_pre) P.i_pre[ob + kl] = (uint8_t)(my_route >> 8);
                 if (P.i_dec) P.i_dec[ob + kl] = (uint8_t)(my_route & 0xFF);
             }
         }
         // drain: every remaining event
-        if (!__any_sync(kFull, err != CTR_OK) && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob, h);
+        if (live && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob, h);
 
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off);
+        for (int off = G / 2; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off, G);
         int status = CTR_OK;
-        if (__any_sync(kFull, err == CTR_ETIMEOUT)) status = CTR_ETIMEOUT;
-        if (__any_sync(kFull, err == CTR_EOVERFLOW)) status = CTR_EOVERFLOW;
-        if (__any_sync(kFull, err == CTR_EINVAL)) status = CTR_EINVAL;
-        if (lane == 0) {
+        if (__ballot_sync(kFull, err == CTR_ETIMEOUT) & gmask) status = CTR_ETIMEOUT;
+        if (__ballot_sync(kFull, err == CTR_EOVERFLOW) & gmask) status = CTR_EOVERFLOW;
+        if (has_row && !valid) status = CTR_EINVAL;
+        if (gl == 0 && has_row) {
             P.row_status[row] = status;
             P.row_hash[row] = status == CTR_OK ? h : 0;
         }
@@ -428,13 +471,25 @@ int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wa
     return (c + 255) / 256 * 256;
 }
 
+int sim_group_width(int n_instances)
+{
+    return n_instances <= 4 ? 4 : n_instances <= 8 ? 8 : n_instances <= 16 ? 16 : 32;
+}
+
 int sim_max_resident_warps(int* warps_per_block, int* blocks)
 {
-    int dev = 0, sms = 0, per_sm = 0;
+    int dev = 0, sms = 0, per_sm = 0, per_sm_g = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sim_kernel, kWarpsPerBlock * 32, 0) != cudaSuccess)
-        return 0;
+    // the smallest occupancy over the group widths, so one workspace size fits every launch
+    per_sm = 1 << 30;
+    const void* kernels[4] = {(const void*)sim_kernel<4>, (const void*)sim_kernel<8>, (const void*)sim_kernel<16>,
+                              (const void*)sim_kernel<32>};
+    for (const void* k : kernels) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_g, k, kWarpsPerBlock * 32, 0) != cudaSuccess)
+            return 0;
+        if (per_sm_g < per_sm) per_sm = per_sm_g;
+    }
     *warps_per_block = kWarpsPerBlock;
     *blocks = sms * per_sm;
     return sms * per_sm * kWarpsPerBlock;
@@ -443,7 +498,12 @@ int sim_max_resident_warps(int* warps_per_block, int* blocks)
 cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
 {
     (void)warps_per_block;
-    sim_kernel<<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
+    switch (sim_group_width(p.n_pre + p.n_dec)) {
+    case 4: sim_kernel<4><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
+    case 8: sim_kernel<8><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
+    case 16: sim_kernel<16><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
+    default: sim_kernel<32><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
+    }
     return cudaGetLastError();
 }
 
