@@ -2,13 +2,13 @@
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
 ``--impl reference`` legs of ``bench.py`` may import this package.  It wraps
-``ctr_oracle.c`` (plain single-threaded C, fp64 / int64) with ctypes and numpy
+``ctr_oracle.c`` (plain single-threaded C, int64, fp64 scorer) with ctypes and numpy
 and shares no code with the CUDA library: configurations arrive as plain
 attribute objects (the workload presets) and are converted here into the
 oracle's own C structs.
 
 Functions follow the paper's sections as cited in ``ctr_oracle.c``:
-Philox4x32-10 and the deterministic fp64 functions, the synthetic trace,
+Philox4x32-10 and the deterministic fp32 functions, the synthetic trace,
 the event-heap simulator (sec. III-A cost, Algorithm 1, sec. III-D, sec. VI
 batching, sec. IV-C baselines), SLO goodput / P99 TTFT, and the fp64
 brute-force scorer.
@@ -93,8 +93,10 @@ def lib():
             build()
             L = C.CDLL(_LIB_PATH)
             L.orc_philox4x32_10.argtypes = [C.POINTER(C.c_uint32), C.POINTER(C.c_uint32), C.POINTER(C.c_uint32)]
-            for name in ("orc_det_log_v", "orc_det_exp_v", "orc_det_ndtri_v"):
-                getattr(L, name).argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_double), C.c_int64]
+            for name in ("orc_det_logf_v", "orc_det_expf_v"):
+                getattr(L, name).argtypes = [C.POINTER(C.c_float), C.POINTER(C.c_float), C.c_int64]
+            for name in ("orc_det_ndtrif_v", "orc_unit_uniform_v"):
+                getattr(L, name).argtypes = [C.POINTER(C.c_uint32), C.POINTER(C.c_float), C.c_int64]
             L.orc_gen_trace.argtypes = [C.POINTER(_TraceCfg), C.c_int64, C.c_int64, C.POINTER(C.c_int64),
                                         C.POINTER(C.c_int32), C.POINTER(C.c_int32), C.POINTER(C.c_int32),
                                         C.POINTER(C.c_uint8)]
@@ -180,23 +182,38 @@ def philox4x32_10(ctr, key):
     return out
 
 
-def _vec(name, x):
-    x = np.ascontiguousarray(x, dtype=np.float64)
+def _vecf(name, x):
+    x = np.ascontiguousarray(x, dtype=np.float32)
     y = np.empty_like(x)
-    getattr(lib(), name)(_p(x, C.c_double), _p(y, C.c_double), x.size)
+    getattr(lib(), name)(_p(x, C.c_float), _p(y, C.c_float), x.size)
     return y
 
 
-def det_log(x):
-    return _vec("orc_det_log_v", x)
+def _vecu(name, u):
+    u = np.ascontiguousarray(u, dtype=np.uint32)
+    y = np.empty(u.shape, np.float32)
+    getattr(lib(), name)(_p(u, C.c_uint32), _p(y, C.c_float), u.size)
+    return y
 
 
-def det_exp(x):
-    return _vec("orc_det_exp_v", x)
+def det_logf(x):
+    """fp32 natural log of the trace construction."""
+    return _vecf("orc_det_logf_v", x)
 
 
-def det_ndtri(x):
-    return _vec("orc_det_ndtri_v", x)
+def det_expf(x):
+    """fp32 exp of the trace construction."""
+    return _vecf("orc_det_expf_v", x)
+
+
+def det_ndtrif(u):
+    """fp32 normal quantile of the uniform (u + 1/2) 2^-32 of a 32-bit word."""
+    return _vecu("orc_det_ndtrif_v", u)
+
+
+def unit_uniform(u):
+    """(u + 1/2) 2^-32 rounded once to fp32."""
+    return _vecu("orc_unit_uniform_v", u)
 
 
 # ---------------------------------------------------------------- trace

@@ -7,10 +7,12 @@
  * product path (the CUDA library under paper_2609_16206_gb300/) never does,
  * and this file shares no code, header, table or constant generator with it.
  *
- * Plain, slow, single-threaded, fp64 / int64, written for checking by eye:
+ * Plain, slow, single-threaded, int64 (fp64 for the scorer), written for
+ * checking by eye:
  *   - Philox4x32-10 counter-based generator (Salmon et al., SC'11, sec. 3).
- *   - Deterministic fp64 log / exp (argument reduction + series) and the
- *     normal quantile of Wichura, Applied Statistics AS241 (PPND16, 1988).
+ *   - Deterministic fp32 log / exp (argument reduction + series) and the
+ *     normal quantile of Wichura, Applied Statistics AS241 (PPND16, 1988),
+ *     the precision in which the trace's integer decisions are defined.
  *   - The synthetic request trace: lognormal prompt / output lengths, a noisy
  *     output-length prediction (sec. III-C) and Poisson or two-state
  *     Markov-modulated Poisson arrivals, all in integer microseconds.
@@ -73,122 +75,120 @@ void orc_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint3
 }
 
 /* ======================================================================
- * Deterministic fp64 elementary functions.  Only +, -, *, / and sqrt, each
- * correctly rounded by IEEE 754, in a fixed order (built with
- * -ffp-contract=off so no product is fused into an FMA).  [reading: the
- * paper fixes no numerics for its trace; the spec fixes these.]
+ * Deterministic fp32 elementary functions.  The trace's floating point only
+ * decides integers (lengths, gaps), so it is defined in the kernel's
+ * precision, fp32: only +, -, *, / and sqrt, each correctly rounded by IEEE
+ * 754, in a fixed order (built with -ffp-contract=off so nothing is fused).
+ * [reading: the paper fixes no numerics for its trace.]
  * ==================================================================== */
-static double bits_to_f64(uint64_t b) { double d; memcpy(&d, &b, 8); return d; }
-static uint64_t f64_to_bits(double d) { uint64_t b; memcpy(&b, &d, 8); return b; }
+static float bits_to_f32(uint32_t b) { float f; memcpy(&f, &b, 4); return f; }
+static uint32_t f32_to_bits(float f) { uint32_t b; memcpy(&b, &f, 4); return b; }
 
-/* ln 2 split for Cody-Waite reduction: HI carries 32 significant bits, so
- * e * HI is exact for |e| < 2^20; LO is the rounded remainder. */
-static const double ORC_LN2_HI = 0x1.62e42fee00000p-1;
-static const double ORC_LN2_LO = 0x1.a39ef35793c76p-33;
-static const double ORC_INV_LN2 = 0x1.71547652b82fep+0;
-static const double ORC_SQRT2 = 0x1.6a09e667f3bcdp+0;
+/* ln 2 split for Cody-Waite reduction: HI carries 16 significant bits, so
+ * e * HI is exact for |e| < 2^8; LO is the rounded remainder. */
+static const float ORC_LN2_HI = 0x1.62e4p-1f;
+static const float ORC_LN2_LO = 0x1.7f7d1cp-20f;
+static const float ORC_INV_LN2 = 0x1.715476p+0f;
+static const float ORC_SQRT2 = 0x1.6a09e6p+0f;
 
 /* log: x = m * 2^e with m in (sqrt(1/2), sqrt(2)]; with s = (m-1)/(m+1),
- * ln m = 2 atanh s = 2 s * sum_{i>=0} s^(2i) / (2i+1), truncated after i = 10
- * (|s| <= 0.1716, so the next term is below 1e-18 of the sum). */
-double orc_det_log(double x)
+ * ln m = 2 s * sum_{i=0..5} s^(2i) / (2i+1) (|s| <= 0.1716: the next term is
+ * below 2^-26 of the sum). */
+float orc_det_logf(float x)
 {
-    static const double inv_odd[11] = {
-        0x1.0000000000000p+0, 0x1.5555555555555p-2, 0x1.999999999999ap-3, 0x1.2492492492492p-3,
-        0x1.c71c71c71c71cp-4, 0x1.745d1745d1746p-4, 0x1.3b13b13b13b14p-4, 0x1.1111111111111p-4,
-        0x1.e1e1e1e1e1e1ep-5, 0x1.af286bca1af28p-5, 0x1.8618618618618p-5};
-    uint64_t b = f64_to_bits(x);
-    int64_t e = (int64_t)((b >> 52) & 0x7ff) - 1023;
-    double m = bits_to_f64((b & 0x000FFFFFFFFFFFFFull) | 0x3FF0000000000000ull);
+    static const float inv_odd[6] = {0x1p+0f, 0x1.555556p-2f, 0x1.99999ap-3f, 0x1.24924ap-3f, 0x1.c71c72p-4f,
+                                     0x1.745d18p-4f};
+    uint32_t b = f32_to_bits(x);
+    int32_t e = (int32_t)((b >> 23) & 0xffu) - 127;
+    float m = bits_to_f32((b & 0x007FFFFFu) | 0x3F800000u);
     if (m > ORC_SQRT2) {
-        m = m * 0.5;
+        m = m * 0.5f;
         e = e + 1;
     }
-    double f = m - 1.0;
-    double s = f / (m + 1.0);
-    double z = s * s;
-    double poly = inv_odd[10];
-    for (int i = 9; i >= 0; --i) poly = poly * z + inv_odd[i];
-    double log_m = (s + s) * poly;
-    double ed = (double)e;
+    float f = m - 1.0f;
+    float s = f / (m + 1.0f);
+    float z = s * s;
+    float poly = inv_odd[5];
+    for (int i = 4; i >= 0; --i) poly = poly * z + inv_odd[i];
+    float log_m = (s + s) * poly;
+    float ed = (float)e;
     return ed * ORC_LN2_HI + (ed * ORC_LN2_LO + log_m);
 }
 
-/* exp: x = k ln2 + r with k = nearest integer to x / ln2, |r| <= ln2 / 2;
- * e^r by its Taylor series to degree 13 (remainder below 5e-18), then scaled
- * by 2^k through the exponent field.  The argument is clamped to [-700, 700]. */
-double orc_det_exp(double x)
+/* exp: x = k ln2 + r with k = nearest integer to x / ln2 (halves away from
+ * zero), |r| <= ln2 / 2; e^r by its Taylor series to degree 7 (remainder
+ * below 2^-27), scaled by 2^k through the exponent field; x clamped to
+ * [-87, 88] so 2^k stays a normal number. */
+float orc_det_expf(float x)
 {
-    static const double inv_fact[14] = {
-        0x1.0000000000000p+0, 0x1.0000000000000p+0, 0x1.0000000000000p-1, 0x1.5555555555555p-3,
-        0x1.5555555555555p-5, 0x1.1111111111111p-7, 0x1.6c16c16c16c17p-10, 0x1.a01a01a01a01ap-13,
-        0x1.a01a01a01a01ap-16, 0x1.71de3a556c734p-19, 0x1.27e4fb7789f5cp-22, 0x1.ae64567f544e4p-26,
-        0x1.1eed8eff8d898p-29, 0x1.6124613a86d09p-33};
-    if (x > 700.0) x = 700.0;
-    if (x < -700.0) x = -700.0;
-    double kf = x * ORC_INV_LN2;
-    int64_t k = (int64_t)(kf >= 0.0 ? kf + 0.5 : kf - 0.5);
-    double kd = (double)k;
-    double r = (x - kd * ORC_LN2_HI) - kd * ORC_LN2_LO;
-    double poly = inv_fact[13];
-    for (int i = 12; i >= 0; --i) poly = poly * r + inv_fact[i];
-    return poly * bits_to_f64((uint64_t)(k + 1023) << 52);
+    static const float inv_fact[8] = {0x1p+0f, 0x1p+0f, 0x1p-1f, 0x1.555556p-3f, 0x1.555556p-5f, 0x1.111112p-7f,
+                                      0x1.6c16c2p-10f, 0x1.a01a02p-13f};
+    if (x > 88.0f) x = 88.0f;
+    if (x < -87.0f) x = -87.0f;
+    float kf = x * ORC_INV_LN2;
+    int32_t k = (int32_t)(kf >= 0.0f ? kf + 0.5f : kf - 0.5f);
+    float kd = (float)k;
+    float r = (x - kd * ORC_LN2_HI) - kd * ORC_LN2_LO;
+    float poly = inv_fact[7];
+    for (int i = 6; i >= 0; --i) poly = poly * r + inv_fact[i];
+    return poly * bits_to_f32((uint32_t)(k + 127) << 23);
 }
 
-/* Normal quantile, Wichura (1988) AS241 PPND16: a degree-7 rational
- * function of r = 0.180625 - q^2 for |q| = |u - 1/2| <= 0.425, otherwise of
- * r = sqrt(-ln min(u, 1-u)) shifted by 1.6 (r <= 5) or by 5. */
-static const double AS241_A[8] = {
-    0x1.b18d91e9eef75p+1, 0x1.0a4888b1a436ep+7, 0x1.ece5d2213c0ccp+10, 0x1.ad1d8cd4ee71dp+13,
-    0x1.66c3e869b752ap+15, 0x1.06c1c55b78f20p+16, 0x1.052d26b2e45e4p+15, 0x1.39a296f7d925ep+11};
-static const double AS241_B[8] = {
-    0x1.0000000000000p+0, 0x1.5281b386e1ab5p+5, 0x1.5797efdc8b3f7p+9, 0x1.512322e75c89fp+12,
-    0x1.4b772d5d65266p+14, 0x1.3317caa64f4bep+15, 0x1.c0e457cb1ae76p+14, 0x1.46a7eca984b69p+12};
-static const double AS241_C[8] = {
-    0x1.6c665fde9526ap+0, 0x1.2857748cab19bp+2, 0x1.713f71462256ap+2, 0x1.d2ecb1a3d02c4p+1,
-    0x1.453cc085375b2p+0, 0x1.ef2abb9b85c37p-3, 0x1.744eb6c45ec67p-6, 0x1.9615ac0b7ace9p-11};
-static const double AS241_D[8] = {
-    0x1.0000000000000p+0, 0x1.06cefbb46a449p+1, 0x1.ad278e6526633p+0, 0x1.61292f23385c9p-1,
-    0x1.2f5123394f040p-3, 0x1.f207a7eab17bfp-7, 0x1.1f18cbfdf2728p-11, 0x1.20d3f686439e4p-30};
-static const double AS241_E[8] = {
-    0x1.aa1b1c13ee526p+2, 0x1.5daea6e875003p+2, 0x1.c8ea6461fa445p+0, 0x1.2fad9315255cfp-2,
-    0x1.b2b41193b4ee7p-6, 0x1.45c1908425345p-10, 0x1.c6ec6cc59e02ap-16, 0x1.afb74d693bf93p-23};
-static const double AS241_F[8] = {
-    0x1.0000000000000p+0, 0x1.331d34fc7d77fp-1, 0x1.186eb183443fbp-3, 0x1.e76f93215462ap-7,
-    0x1.9c8bc979dc5d7p-11, 0x1.35c2c496374bfp-16, 0x1.31446f740b9e0p-23, 0x1.269bff1f8c190p-49};
+/* The uniform of a 32-bit word: (u + 1/2) 2^-32, rounded once to fp32.  Its
+ * complement 1 - U is the same construction applied to ~u, so a tail never
+ * needs a cancelling subtraction. */
+float orc_unit_uniform(uint32_t u) { return (float)(int64_t)(2 * (uint64_t)u + 1) * 0x1p-33f; }
 
-static double horner7(const double c[8], double r)
+/* Normal quantile of U(u), Wichura (1988) AS241 PPND16 evaluated in fp32: a
+ * degree-7 rational function of r = 0.180625 - q^2 for |q| = |U - 1/2| <= 0.425,
+ * otherwise of r = sqrt(-ln min(U, 1-U)) shifted by 1.6 (r <= 5) or by 5. */
+static const float AS241_A[8] = {0x1.b18d92p+1f, 0x1.0a4888p+7f, 0x1.ece5d2p+10f, 0x1.ad1d8cp+13f,
+                                 0x1.66c3e8p+15f, 0x1.06c1c6p+16f, 0x1.052d26p+15f, 0x1.39a296p+11f};
+static const float AS241_B[8] = {0x1p+0f, 0x1.5281b4p+5f, 0x1.5797fp+9f, 0x1.512322p+12f,
+                                 0x1.4b772ep+14f, 0x1.3317cap+15f, 0x1.c0e458p+14f, 0x1.46a7ecp+12f};
+static const float AS241_C[8] = {0x1.6c666p+0f, 0x1.285774p+2f, 0x1.713f72p+2f, 0x1.d2ecb2p+1f,
+                                 0x1.453ccp+0f, 0x1.ef2abcp-3f, 0x1.744eb6p-6f, 0x1.9615acp-11f};
+static const float AS241_D[8] = {0x1p+0f, 0x1.06cefcp+1f, 0x1.ad278ep+0f, 0x1.61293p-1f,
+                                 0x1.2f5124p-3f, 0x1.f207a8p-7f, 0x1.1f18ccp-11f, 0x1.20d3f6p-30f};
+static const float AS241_E[8] = {0x1.aa1b1cp+2f, 0x1.5daea6p+2f, 0x1.c8ea64p+0f, 0x1.2fad94p-2f,
+                                 0x1.b2b412p-6f, 0x1.45c19p-10f, 0x1.c6ec6cp-16f, 0x1.afb74ep-23f};
+static const float AS241_F[8] = {0x1p+0f, 0x1.331d34p-1f, 0x1.186eb2p-3f, 0x1.e76f94p-7f,
+                                 0x1.9c8bcap-11f, 0x1.35c2c4p-16f, 0x1.31447p-23f, 0x1.269cp-49f};
+
+static float horner7(const float c[8], float r)
 {
-    double acc = c[7];
+    float acc = c[7];
     for (int i = 6; i >= 0; --i) acc = acc * r + c[i];
     return acc;
 }
 
-double orc_det_ndtri(double u)
+float orc_det_ndtrif(uint32_t u)
 {
-    double q = u - 0.5;
-    double aq = q < 0.0 ? -q : q;
-    if (aq <= 0x1.b333333333333p-2 /* 0.425 */) {
-        double r = 0x1.71eb851eb851fp-3 /* 0.180625 */ - q * q;
+    int64_t c = 2 * (int64_t)u + 1 - 4294967296LL; /* 2^33 (U - 1/2), odd, never 0 */
+    float q = (float)c * 0x1p-33f;
+    float aq = q < 0.0f ? -q : q;
+    if (aq <= 0x1.b33334p-2f /* 0.425 */) {
+        float r = 0x1.71eb86p-3f /* 0.180625 */ - q * q;
         return (q * horner7(AS241_A, r)) / horner7(AS241_B, r);
     }
-    double tail = q < 0.0 ? u : 1.0 - u;
-    double r = sqrt(-orc_det_log(tail));
-    double v;
-    if (r <= 5.0) {
-        r = r - 0x1.999999999999ap+0; /* 1.6 */
+    float tail = c < 0 ? orc_unit_uniform(u) : orc_unit_uniform(~u);
+    float r = sqrtf(-orc_det_logf(tail));
+    float v;
+    if (r <= 5.0f) {
+        r = r - 0x1.99999ap+0f; /* 1.6 */
         v = horner7(AS241_C, r) / horner7(AS241_D, r);
     } else {
-        r = r - 5.0;
+        r = r - 5.0f;
         v = horner7(AS241_E, r) / horner7(AS241_F, r);
     }
-    return q < 0.0 ? -v : v;
+    return c < 0 ? -v : v;
 }
 
 /* vectorised entry points for the pin tests */
-void orc_det_log_v(const double* x, double* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_det_log(x[i]); }
-void orc_det_exp_v(const double* x, double* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_det_exp(x[i]); }
-void orc_det_ndtri_v(const double* x, double* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_det_ndtri(x[i]); }
+void orc_det_logf_v(const float* x, float* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_det_logf(x[i]); }
+void orc_det_expf_v(const float* x, float* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_det_expf(x[i]); }
+void orc_det_ndtrif_v(const uint32_t* u, float* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_det_ndtrif(u[i]); }
+void orc_unit_uniform_v(const uint32_t* u, float* y, int64_t n) { for (int64_t i = 0; i < n; ++i) y[i] = orc_unit_uniform(u[i]); }
 
 /* ======================================================================
  * Synthetic trace (the workloads of Table 1 as length laws; sec. III-C
@@ -213,12 +213,11 @@ typedef struct {
     uint64_t class_thr[3];    /* cumulative class probabilities * 2^32 */
 } orc_trace_cfg;
 
-static double unit_uniform(uint32_t x) { return ((double)x + 0.5) * 0x1p-32; }
-
-static int64_t round_clip(double e, int64_t lo, int64_t hi)
+/* clip(floor(v + 1/2), lo, hi) for v >= 0 (NaN / inf / huge -> hi) */
+static int64_t round_clip(float v, int64_t lo, int64_t hi)
 {
-    double y = e + 0.5;
-    if (!(y < (double)hi)) return hi;
+    float y = v + 0.5f;
+    if (!(y < (float)hi)) return hi;
     int64_t t = (int64_t)y;
     return t < lo ? lo : t;
 }
@@ -237,8 +236,8 @@ static int64_t dwell_us(const orc_trace_cfg* cfg, uint64_t sub, uint64_t j)
 {
     uint32_t x[4];
     draw(cfg, sub, 1u, j, 0u, x);
-    double g = orc_det_log(unit_uniform(x[0]));
-    return (int64_t)((-g) * (double)cfg->dwell_mean_us);
+    float g = orc_det_logf(orc_unit_uniform(x[0]));
+    return (int64_t)((-g) * (float)cfg->dwell_mean_us);
 }
 
 /* One replica (global index g) of n requests, written to the five arrays. */
@@ -263,24 +262,25 @@ int orc_gen_trace(const orc_trace_cfg* cfg_in, int64_t g, int64_t n, int64_t* ar
         draw(&cfg, sub, 0u, (uint64_t)k, 0u, x);
         draw(&cfg, sub, 0u, (uint64_t)k, 1u, y);
 
-        double zp = orc_det_ndtri(unit_uniform(x[0]));
-        int64_t p = round_clip(orc_det_exp(cfg.prompt_mu + cfg.prompt_sigma * zp), cfg.prompt_min, cfg.prompt_max);
+        float zp = orc_det_ndtrif(x[0]);
+        int64_t p = round_clip(orc_det_expf((float)cfg.prompt_mu + (float)cfg.prompt_sigma * zp), cfg.prompt_min,
+                               cfg.prompt_max);
 
         int is_short = (uint64_t)x[1] < cfg.mix_short_thr;
-        double mu = is_short ? cfg.short_mu : cfg.long_mu;
-        double sg = is_short ? cfg.short_sigma : cfg.long_sigma;
-        double zo = orc_det_ndtri(unit_uniform(x[2]));
-        int64_t o = round_clip(orc_det_exp(mu + sg * zo), cfg.out_min, cfg.out_max);
+        float mu = is_short ? (float)cfg.short_mu : (float)cfg.long_mu;
+        float sg = is_short ? (float)cfg.short_sigma : (float)cfg.long_sigma;
+        float zo = orc_det_ndtrif(x[2]);
+        int64_t o = round_clip(orc_det_expf(mu + sg * zo), cfg.out_min, cfg.out_max);
 
-        double zn = orc_det_ndtri(unit_uniform(x[3]));
-        double factor = orc_det_exp(cfg.noise_sigma * zn);
-        int64_t oh = round_clip((double)o * factor, cfg.pred_min, cfg.pred_max);
+        float zn = orc_det_ndtrif(x[3]);
+        float factor = orc_det_expf((float)cfg.noise_sigma * zn);
+        int64_t oh = round_clip((float)o * factor, cfg.pred_min, cfg.pred_max);
 
         int64_t c = 0;
         while (c < cfg.n_classes - 1 && (uint64_t)y[0] >= cfg.class_thr[c]) c++;
 
-        double lg = orc_det_log(unit_uniform(y[1]));
-        int64_t gap = (int64_t)((-lg) * 1e9);
+        float lg = orc_det_logf(orc_unit_uniform(y[1]));
+        int64_t gap = (int64_t)((-lg) * 0x1.dcd65p+29f /* 1e9 */);
         lambda += gap;
 
         int64_t t;

@@ -111,14 +111,17 @@ int ctr_gen_trace(const ctr_trace_cfg* cfg, int32_t n_replicas, int64_t replica_
     p.n_classes = cfg->n_classes;
     p.rate[0] = cfg->rate_mreq[0];
     p.rate[1] = cfg->rate_mreq[1];
+    p.rate_recip[0] = ~0ull / (uint64_t)cfg->rate_mreq[0];
+    p.rate_recip[1] = ~0ull / (uint64_t)cfg->rate_mreq[1];
     p.dwell_mean_us = cfg->dwell_mean_us;
-    p.prompt_mu = cfg->prompt_mu;
-    p.prompt_sigma = cfg->prompt_sigma;
-    p.short_mu = cfg->short_mu;
-    p.short_sigma = cfg->short_sigma;
-    p.long_mu = cfg->long_mu;
-    p.long_sigma = cfg->long_sigma;
-    p.noise_sigma = cfg->noise_sigma;
+    // the trace is defined in fp32: each parameter is rounded once from the caller's double
+    p.prompt_mu = (float)cfg->prompt_mu;
+    p.prompt_sigma = (float)cfg->prompt_sigma;
+    p.short_mu = (float)cfg->short_mu;
+    p.short_sigma = (float)cfg->short_sigma;
+    p.long_mu = (float)cfg->long_mu;
+    p.long_sigma = (float)cfg->long_sigma;
+    p.noise_sigma = (float)cfg->noise_sigma;
     p.prompt_min = cfg->prompt_min;
     p.prompt_max = cfg->prompt_max;
     p.out_min = cfg->out_min;

@@ -22,8 +22,9 @@ struct TraceParams {
     int32_t arrival_kind;
     int32_t n_classes;
     int64_t rate[2];
+    uint64_t rate_recip[2];     // floor((2^64 - 1) / rate)
     int64_t dwell_mean_us;
-    double prompt_mu, prompt_sigma, short_mu, short_sigma, long_mu, long_sigma, noise_sigma;
+    float prompt_mu, prompt_sigma, short_mu, short_sigma, long_mu, long_sigma, noise_sigma;
     int64_t prompt_min, prompt_max, out_min, out_max, pred_min, pred_max;
     uint64_t mix_short_thr;
     uint64_t class_thr[3];

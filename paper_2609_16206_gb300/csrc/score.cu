@@ -8,18 +8,22 @@
 // a_d^s + m_d^s * o_hat with a_d^s = sigma_s w_b backlog_d + w_q A_d and
 // m_d^s = sigma_s w_s tau_dec rho kappa_d >= 0.  Each block stages the
 // instance state into shared memory with a TMA bulk copy (cp.async.bulk +
-// mbarrier), builds the four per-class envelopes (one thread per (class,
-// line): the interval of o_hat on which the line wins, then its rank), and
-// streams requests with 128-bit loads: a binary search over the envelope's
-// breakpoints gives the argmin, whose fp32 cost is then evaluated from the
-// full formula.  The work per request is O(log envelope size) instead of
-// O(instances), which keeps the kernel on the HBM roofline.
+// mbarrier) while its first request vectors are already in flight, builds the
+// four per-class envelopes (one thread per (class, line): a division-free
+// Pareto test -- a line with both a larger intercept and a larger slope than
+// another can never win -- then, for the few surviving lines, the interval of
+// o_hat on which the line wins and its rank), and streams requests with
+// 128-bit loads, software-pipelined one vector ahead: a binary search over the
+// envelope's breakpoints gives the argmin, whose fp32 cost is then evaluated
+// from the full formula.  The work per request is O(log envelope size) instead
+// of O(instances), which keeps the kernel on the HBM roofline.  One block per
+// SM, so the envelope is built 152 times, not once per request tile.
 #include "ctr_internal.cuh"
 
 namespace ctr {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 1024;
 constexpr int kMaxInst = CTR_SCORE_MAX_INST;
 constexpr unsigned kWaitLimit = 1u << 22;  // bounded mbarrier polling
 
@@ -29,8 +33,11 @@ struct __align__(16) Smem {
     float kap[kMaxInst];
     float bk[kMaxInst];   // w_b * (tau_pre Q + tau_act A)
     float wqa[kMaxInst];  // w_q * A
+    float la[4][kMaxInst];   // line intercept per class
+    float lm[4][kMaxInst];   // line slope (per unit o_hat) per class
     float lo_tmp[4][kMaxInst];
     int valid_tmp[4][kMaxInst];
+    int pareto[4][kMaxInst];
     float seg_lo[4][kMaxInst];
     int seg_id[4][kMaxInst];
     int nseg[4];
@@ -97,12 +104,28 @@ __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, 
 }
 
 template <bool kVec>
-__global__ void __launch_bounds__(kThreads) score_kernel(const ScoreParams P)
+__global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
 {
     extern __shared__ __align__(128) unsigned char smem_raw[];
     Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
     const int tid = threadIdx.x;
     const int n_inst = P.n_inst;
+
+    // first request vector of this thread, in flight while the block builds its envelopes
+    const int64_t nv = kVec ? (P.n >> 2) : 0;
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    int64_t v = (int64_t)blockIdx.x * kThreads + tid;
+    bool has = kVec && v < nv;
+    const float4* p4 = reinterpret_cast<const float4*>(P.p);
+    const float4* o4 = reinterpret_cast<const float4*>(P.oh);
+    const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
+    float4 pv = make_float4(0.f, 0.f, 0.f, 0.f), ov = pv;
+    uint32_t cv = 0;
+    if (has) {
+        pv = ld_stream(p4 + v);
+        ov = ld_stream(o4 + v);
+        cv = ld_stream_u32(c4 + v);
+    }
 
     // ---- stage the instance state: TMA bulk copy when aligned, else plain loads
     const uint32_t bytes = (uint32_t)n_inst * 4u;
@@ -140,11 +163,9 @@ __global__ void __launch_bounds__(kThreads) score_kernel(const ScoreParams P)
                 : "r"(bar)
                 : "memory");
         }
-        if (!done) {
-            // never expected: report, then read the state directly; the block
-            // still waits (bounded) above for its own copies before exiting
-            if (P.status) atomicExch(P.status, CTR_ETIMEOUT);
-            __syncthreads();
+        if (__syncthreads_or(!done)) {  // block-uniform decision
+            // never expected: report it and read the state with plain loads instead
+            if (tid == 0 && P.status) atomicExch(P.status, CTR_ETIMEOUT);
             for (int d = tid; d < n_inst; d += kThreads) {
                 sm.q[d] = P.Q[d];
                 sm.a[d] = P.A[d];
@@ -165,26 +186,42 @@ __global__ void __launch_bounds__(kThreads) score_kernel(const ScoreParams P)
     }
     __syncthreads();
 
-    // ---- per-class lower envelope: the o_hat interval on which each line wins
+    // ---- per-class lower envelope
     for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {
         const int s = idx / n_inst, d = idx - s * n_inst;
-        float ad, md;
-        line_of(sm, P, s, d, ad, md);
-        float lo = 0.0f, hi = __int_as_float(0x7f800000);
-        bool empty = false;
+        line_of(sm, P, s, d, sm.la[s][d], sm.lm[s][d]);
+    }
+    __syncthreads();
+    for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {  // Pareto filter (ties: lowest index survives)
+        const int s = idx / n_inst, d = idx - s * n_inst;
+        const float ad = sm.la[s][d], md = sm.lm[s][d];
+        bool dominated = false;
         for (int e = 0; e < n_inst; ++e) {
-            if (e == d) continue;
-            float ae, me;
-            line_of(sm, P, s, e, ae, me);
-            if (me == md) {
-                if (ae < ad || (ae == ad && e < d)) empty = true;
-            } else if (me > md) {
-                lo = fmaxf(lo, (ad - ae) / (me - md));
-            } else {
-                hi = fminf(hi, (ae - ad) / (md - me));
-            }
+            const float ae = sm.la[s][e], me = sm.lm[s][e];
+            dominated |= ae <= ad && me <= md && (ae < ad || me < md || e < d);
         }
-        sm.valid_tmp[s][d] = !empty && lo < hi;
+        sm.pareto[s][d] = !dominated;
+    }
+    __syncthreads();
+    for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {  // winning o_hat interval of each surviving line
+        const int s = idx / n_inst, d = idx - s * n_inst;
+        bool valid = false;
+        float lo = 0.0f;
+        if (sm.pareto[s][d]) {
+            const float ad = sm.la[s][d], md = sm.lm[s][d];
+            float hi = __int_as_float(0x7f800000);
+            for (int e = 0; e < n_inst; ++e) {
+                if (e == d || !sm.pareto[s][e]) continue;
+                const float ae = sm.la[s][e], me = sm.lm[s][e];
+                if (me > md) {
+                    lo = fmaxf(lo, (ad - ae) / (me - md));
+                } else if (me < md) {
+                    hi = fminf(hi, (ae - ad) / (md - me));
+                }
+            }
+            valid = lo < hi;
+        }
+        sm.valid_tmp[s][d] = valid;
         sm.lo_tmp[s][d] = lo;
     }
     if (tid < 4) sm.nseg[tid] = 0;
@@ -218,18 +255,20 @@ __global__ void __launch_bounds__(kThreads) score_kernel(const ScoreParams P)
     }
     __syncthreads();
 
-    // ---- stream the requests
+    // ---- stream the requests (the first vector was loaded before the prologue)
     if (kVec) {
-        const int64_t nv = P.n >> 2;
-        const float4* p4 = reinterpret_cast<const float4*>(P.p);
-        const float4* o4 = reinterpret_cast<const float4*>(P.oh);
-        const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
         int4* a4 = reinterpret_cast<int4*>(P.argmin);
         float4* f4 = reinterpret_cast<float4*>(P.cost);
-        for (int64_t v = (int64_t)blockIdx.x * kThreads + tid; v < nv; v += (int64_t)gridDim.x * kThreads) {
-            const float4 pv = ld_stream(p4 + v);
-            const float4 ov = ld_stream(o4 + v);
-            const uint32_t cv = ld_stream_u32(c4 + v);
+        while (has) {
+            const int64_t vn = v + stride;
+            const bool hn = vn < nv;
+            float4 pn = make_float4(0.f, 0.f, 0.f, 0.f), on = pn;
+            uint32_t cn = 0;
+            if (hn) {
+                pn = ld_stream(p4 + vn);
+                on = ld_stream(o4 + vn);
+                cn = ld_stream_u32(c4 + vn);
+            }
             int4 ai;
             float4 fc;
             score_one(sm, P, pv.x, ov.x, cv & 0xFFu, ai.x, fc.x);
@@ -238,6 +277,11 @@ __global__ void __launch_bounds__(kThreads) score_kernel(const ScoreParams P)
             score_one(sm, P, pv.w, ov.w, cv >> 24, ai.w, fc.w);
             __stcs(a4 + v, ai);
             __stcs(f4 + v, fc);
+            v = vn;
+            has = hn;
+            pv = pn;
+            ov = on;
+            cv = cn;
         }
         if (blockIdx.x == 0 && tid < (int)(P.n & 3)) {
             const int64_t i = (nv << 2) + tid;
@@ -273,7 +317,7 @@ cudaError_t launch_score(const ScoreParams& p, cudaStream_t stream)
     const int smem = (int)sizeof(Smem);
     const int64_t per_block = vec ? 4 * kThreads : kThreads;
     int64_t blocks = (p.n + per_block - 1) / per_block;
-    const int64_t cap = (int64_t)sms * 4;
+    const int64_t cap = (int64_t)sms;
     if (blocks > cap) blocks = cap;
     if (vec) {
         err = cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);

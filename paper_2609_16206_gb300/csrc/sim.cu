@@ -37,6 +37,7 @@ constexpr int kWarpsPerBlock = 4;
 constexpr int64_t kNever = INT64_MAX;
 constexpr int64_t kBacklogClamp = int64_t(1) << 40;
 constexpr int64_t kPressureClamp = int64_t(1) << 18;
+constexpr int kRecipN = 1024;  // batch sizes with a tabulated reciprocal
 
 __device__ __forceinline__ uint64_t mix64(uint64_t z)  // splitmix64 output function
 {
@@ -134,8 +135,23 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                                               uint32_t* wait, int64_t tb, int64_t ob, uint64_t& h)
 {
     for (;;) {
-        const int64_t te = s.stepping ? s.step_end : kNever;
+        // Plain step ends first, in a tight loop: the step ends by T, no request
+        // finishes with it, nothing becomes KV-ready at that instant and nobody
+        // waits for admission, so the batch is unchanged and the next step
+        // starts at once.  Lanes leave this loop at their next non-plain event;
+        // the general handler below then runs once for all of them together.
         const int64_t tp = s.pend_n > 0 ? (int64_t)(s.pend_top >> kKeyBits) : kNever;
+        const int64_t limit = tp <= T ? tp - 1 : T;  // plain step ends lie at or before limit
+        while (s.stepping && s.step_end <= limit && s.w_n == 0 &&
+               (int64_t)(s.act_top >> kKeyBits) != s.step_idx + 1) {
+            s.step_idx += 1;
+            s.kv_res += s.n_act;
+            s.R -= s.n_act;
+            if (++s.steps > P.max_steps) return CTR_ETIMEOUT;
+            s.step_end += P.dec_base + P.dec_seq * s.n_act + kv_term(s.kv_res, P);
+            if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
+        }
+        const int64_t te = s.stepping ? s.step_end : kNever;
         const int64_t tev = te < tp ? te : tp;
         if (tev > T) return CTR_OK;
         if (te == tev) {  // (1) the running step ends: one token for every active request
@@ -259,9 +275,13 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // the per-lane event loops, the per-group argmins and the commits are
 // independent across groups.
 template <int G>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_constant__ SimParams P)
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, 4) sim_kernel(const __grid_constant__ SimParams P)
 {
     constexpr int kRowsPerWarp = 32 / G;
+    // floor((2^64 - 1) / n) for the decode backlog's division by the batch size
+    __shared__ uint64_t recip[kRecipN + 1];
+    for (int i = threadIdx.x; i <= kRecipN; i += blockDim.x) recip[i] = i == 0 ? 0 : ~0ull / (uint64_t)i;
+    __syncthreads();
     const int lane = threadIdx.x & 31;
     const int grp = lane / G;
     const int gl = lane % G;
@@ -372,7 +392,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32) sim_kernel(const __grid_c
                             if (hi != 0 || lo >= (1ull << 62)) {
                                 b = kBacklogClamp;
                             } else {
-                                b = (int64_t)(lo / (uint64_t)(na > 1 ? na : 1));
+                                const uint64_t nd = (uint64_t)(na > 1 ? na : 1);
+                                b = (int64_t)(nd <= (uint64_t)kRecipN ? div_recip(lo, nd, recip[nd]) : lo / nd);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
                             int64_t press = (int64_t)div_recip((uint64_t)(s.kv_res + pk + ohk) << 16,

@@ -9,11 +9,12 @@
 // the rate, MMPP arrivals walk the state intervals cooperatively.
 //
 // Bit-identity with the CPU reference construction rests on doing only IEEE
-// basic operations in a fixed order: every fp64 operation below is an
-// explicit round-to-nearest intrinsic (no contraction into FMA; the file is
-// also compiled with -fmad=false), and log / exp / the normal quantile are
-// written here from their published methods rather than taken from CUDA's
-// math library.
+// basic operations in a fixed order, in fp32 (the precision the integer
+// lengths and gaps are defined in; GB300's fp64 rate would bound the kernel):
+// every operation below is an explicit round-to-nearest intrinsic (no
+// contraction into FMA; the file is also compiled with -fmad=false), and
+// log / exp / the normal quantile are written here from their published
+// methods rather than taken from CUDA's math library.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -42,131 +43,134 @@ __device__ __forceinline__ U32x4 philox(uint32_t c0, uint32_t c1, uint32_t c2, u
     return U32x4{{c0, c1, c2, c3}};
 }
 
-// ------------------------------------------------------------- fp64 helpers
-__device__ __forceinline__ double add(double a, double b) { return __dadd_rn(a, b); }
-__device__ __forceinline__ double sub(double a, double b) { return __dsub_rn(a, b); }
-__device__ __forceinline__ double mul(double a, double b) { return __dmul_rn(a, b); }
-__device__ __forceinline__ double dvd(double a, double b) { return __ddiv_rn(a, b); }
+// ------------------------------------------------------------- fp32 helpers
+__device__ __forceinline__ float add(float a, float b) { return __fadd_rn(a, b); }
+__device__ __forceinline__ float sub(float a, float b) { return __fsub_rn(a, b); }
+__device__ __forceinline__ float mul(float a, float b) { return __fmul_rn(a, b); }
+__device__ __forceinline__ float dvd(float a, float b) { return __fdiv_rn(a, b); }
 
-__device__ __forceinline__ double u01(uint32_t x)  // (x + 1/2) 2^-32, exact
+// (u + 1/2) 2^-32 rounded once to fp32; 1 - U is the same of ~u
+__device__ __forceinline__ float u01(uint32_t u)
 {
-    return mul(add(__uint2double_rn(x), 0.5), 0x1p-32);
+    return mul(__ll2float_rn((long long)(2ull * u + 1ull)), 0x1p-33f);
 }
 
-// Natural log for positive normal x: x = m 2^e with m in (sqrt(1/2), sqrt(2)],
-// s = (m - 1)/(m + 1), ln m = 2 s sum_{i=0..10} s^(2i) / (2i + 1) by Horner,
-// ln x = e * ln2_hi + (e * ln2_lo + ln m)  (ln2_hi has 32 significant bits).
-__device__ double det_log(double x)
+// Natural log of a positive normal x: x = m 2^e with m in (sqrt(1/2), sqrt(2)],
+// s = (m - 1)/(m + 1), ln m = 2 s sum_{i=0..5} s^(2i) / (2i + 1) by Horner,
+// ln x = e * ln2_hi + (e * ln2_lo + ln m)  (ln2_hi has 16 significant bits).
+__device__ float det_logf(float x)
 {
-    const double inv_odd[11] = {0x1.0000000000000p+0, 0x1.5555555555555p-2, 0x1.999999999999ap-3,
-                                0x1.2492492492492p-3, 0x1.c71c71c71c71cp-4, 0x1.745d1745d1746p-4,
-                                0x1.3b13b13b13b14p-4, 0x1.1111111111111p-4, 0x1.e1e1e1e1e1e1ep-5,
-                                0x1.af286bca1af28p-5, 0x1.8618618618618p-5};
-    const unsigned long long bits = (unsigned long long)__double_as_longlong(x);
-    long long e = (long long)((bits >> 52) & 0x7ffull) - 1023;
-    double m = __longlong_as_double((long long)((bits & 0x000FFFFFFFFFFFFFull) | 0x3FF0000000000000ull));
-    if (m > 0x1.6a09e667f3bcdp+0) {
-        m = mul(m, 0.5);
+    const float inv_odd[6] = {0x1p+0f, 0x1.555556p-2f, 0x1.99999ap-3f, 0x1.24924ap-3f, 0x1.c71c72p-4f, 0x1.745d18p-4f};
+    const uint32_t bits = __float_as_uint(x);
+    int e = (int)((bits >> 23) & 0xffu) - 127;
+    float m = __uint_as_float((bits & 0x007FFFFFu) | 0x3F800000u);
+    if (m > 0x1.6a09e6p+0f) {
+        m = mul(m, 0.5f);
         e += 1;
     }
-    const double f = sub(m, 1.0);
-    const double s = dvd(f, add(m, 1.0));
-    const double z = mul(s, s);
-    double acc = inv_odd[10];
+    const float f = sub(m, 1.0f);
+    const float s = dvd(f, add(m, 1.0f));
+    const float z = mul(s, s);
+    float acc = inv_odd[5];
 #pragma unroll
-    for (int i = 9; i >= 0; --i) acc = add(mul(acc, z), inv_odd[i]);
-    const double ln_m = mul(add(s, s), acc);
-    const double ed = __ll2double_rn(e);
-    return add(mul(ed, 0x1.62e42fee00000p-1), add(mul(ed, 0x1.a39ef35793c76p-33), ln_m));
+    for (int i = 4; i >= 0; --i) acc = add(mul(acc, z), inv_odd[i]);
+    const float ln_m = mul(add(s, s), acc);
+    const float ed = __int2float_rn(e);
+    return add(mul(ed, 0x1.62e4p-1f), add(mul(ed, 0x1.7f7d1cp-20f), ln_m));
 }
 
 // exp: k = nearest integer to x / ln2 (halves away from zero),
-// r = (x - k ln2_hi) - k ln2_lo, e^r by its degree-13 Taylor polynomial,
-// times 2^k through the exponent field.  x is clamped to [-700, 700].
-__device__ double det_exp(double x)
+// r = (x - k ln2_hi) - k ln2_lo, e^r by its degree-7 Taylor polynomial, times
+// 2^k through the exponent field.  x is clamped to [-87, 88].
+__device__ float det_expf(float x)
 {
-    const double inv_fact[14] = {0x1.0000000000000p+0, 0x1.0000000000000p+0, 0x1.0000000000000p-1,
-                                 0x1.5555555555555p-3, 0x1.5555555555555p-5, 0x1.1111111111111p-7,
-                                 0x1.6c16c16c16c17p-10, 0x1.a01a01a01a01ap-13, 0x1.a01a01a01a01ap-16,
-                                 0x1.71de3a556c734p-19, 0x1.27e4fb7789f5cp-22, 0x1.ae64567f544e4p-26,
-                                 0x1.1eed8eff8d898p-29, 0x1.6124613a86d09p-33};
-    if (x > 700.0) x = 700.0;
-    if (x < -700.0) x = -700.0;
-    const double kf = mul(x, 0x1.71547652b82fep+0);
-    const long long k = __double2ll_rz(kf >= 0.0 ? add(kf, 0.5) : sub(kf, 0.5));
-    const double kd = __ll2double_rn(k);
-    const double r = sub(sub(x, mul(kd, 0x1.62e42fee00000p-1)), mul(kd, 0x1.a39ef35793c76p-33));
-    double acc = inv_fact[13];
+    const float inv_fact[8] = {0x1p+0f, 0x1p+0f, 0x1p-1f, 0x1.555556p-3f, 0x1.555556p-5f, 0x1.111112p-7f,
+                               0x1.6c16c2p-10f, 0x1.a01a02p-13f};
+    if (x > 88.0f) x = 88.0f;
+    if (x < -87.0f) x = -87.0f;
+    const float kf = mul(x, 0x1.715476p+0f);
+    const int k = __float2int_rz(kf >= 0.0f ? add(kf, 0.5f) : sub(kf, 0.5f));
+    const float kd = __int2float_rn(k);
+    const float r = sub(sub(x, mul(kd, 0x1.62e4p-1f)), mul(kd, 0x1.7f7d1cp-20f));
+    float acc = inv_fact[7];
 #pragma unroll
-    for (int i = 12; i >= 0; --i) acc = add(mul(acc, r), inv_fact[i]);
-    return mul(acc, __longlong_as_double((long long)((unsigned long long)(k + 1023) << 52)));
+    for (int i = 6; i >= 0; --i) acc = add(mul(acc, r), inv_fact[i]);
+    return mul(acc, __uint_as_float((uint32_t)(k + 127) << 23));
 }
 
-// Wichura (1988), algorithm AS241 PPND16: rational approximations of degree 7
-// in r = 0.180625 - q^2 (|q| <= 0.425, q = u - 1/2) or in
-// r = sqrt(-ln min(u, 1 - u)) shifted by 1.6 (r <= 5) or by 5.
-__device__ __forceinline__ double poly7(const double* c, double r)
+// Wichura (1988), algorithm AS241 PPND16 in fp32: rational approximations of
+// degree 7 in r = 0.180625 - q^2 (|q| <= 0.425, q = U - 1/2) or in
+// r = sqrt(-ln min(U, 1 - U)) shifted by 1.6 (r <= 5) or by 5.
+__device__ __forceinline__ float poly7(const float* c, float r)
 {
-    double acc = c[7];
+    float acc = c[7];
 #pragma unroll
     for (int i = 6; i >= 0; --i) acc = add(mul(acc, r), c[i]);
     return acc;
 }
 
-__device__ double det_ndtri(double u)
+__device__ float det_ndtrif(uint32_t u)
 {
-    const double a[8] = {0x1.b18d91e9eef75p+1, 0x1.0a4888b1a436ep+7, 0x1.ece5d2213c0ccp+10,
-                         0x1.ad1d8cd4ee71dp+13, 0x1.66c3e869b752ap+15, 0x1.06c1c55b78f20p+16,
-                         0x1.052d26b2e45e4p+15, 0x1.39a296f7d925ep+11};
-    const double b[8] = {0x1.0000000000000p+0, 0x1.5281b386e1ab5p+5, 0x1.5797efdc8b3f7p+9,
-                         0x1.512322e75c89fp+12, 0x1.4b772d5d65266p+14, 0x1.3317caa64f4bep+15,
-                         0x1.c0e457cb1ae76p+14, 0x1.46a7eca984b69p+12};
-    const double c[8] = {0x1.6c665fde9526ap+0, 0x1.2857748cab19bp+2, 0x1.713f71462256ap+2,
-                         0x1.d2ecb1a3d02c4p+1, 0x1.453cc085375b2p+0, 0x1.ef2abb9b85c37p-3,
-                         0x1.744eb6c45ec67p-6, 0x1.9615ac0b7ace9p-11};
-    const double d[8] = {0x1.0000000000000p+0, 0x1.06cefbb46a449p+1, 0x1.ad278e6526633p+0,
-                         0x1.61292f23385c9p-1, 0x1.2f5123394f040p-3, 0x1.f207a7eab17bfp-7,
-                         0x1.1f18cbfdf2728p-11, 0x1.20d3f686439e4p-30};
-    const double e[8] = {0x1.aa1b1c13ee526p+2, 0x1.5daea6e875003p+2, 0x1.c8ea6461fa445p+0,
-                         0x1.2fad9315255cfp-2, 0x1.b2b41193b4ee7p-6, 0x1.45c1908425345p-10,
-                         0x1.c6ec6cc59e02ap-16, 0x1.afb74d693bf93p-23};
-    const double f[8] = {0x1.0000000000000p+0, 0x1.331d34fc7d77fp-1, 0x1.186eb183443fbp-3,
-                         0x1.e76f93215462ap-7, 0x1.9c8bc979dc5d7p-11, 0x1.35c2c496374bfp-16,
-                         0x1.31446f740b9e0p-23, 0x1.269bff1f8c190p-49};
-    const double q = sub(u, 0.5);
-    const double aq = q < 0.0 ? -q : q;
-    if (aq <= 0x1.b333333333333p-2) {
-        const double r = sub(0x1.71eb851eb851fp-3, mul(q, q));
+    const float a[8] = {0x1.b18d92p+1f, 0x1.0a4888p+7f, 0x1.ece5d2p+10f, 0x1.ad1d8cp+13f,
+                        0x1.66c3e8p+15f, 0x1.06c1c6p+16f, 0x1.052d26p+15f, 0x1.39a296p+11f};
+    const float b[8] = {0x1p+0f, 0x1.5281b4p+5f, 0x1.5797fp+9f, 0x1.512322p+12f,
+                        0x1.4b772ep+14f, 0x1.3317cap+15f, 0x1.c0e458p+14f, 0x1.46a7ecp+12f};
+    const float c[8] = {0x1.6c666p+0f, 0x1.285774p+2f, 0x1.713f72p+2f, 0x1.d2ecb2p+1f,
+                        0x1.453ccp+0f, 0x1.ef2abcp-3f, 0x1.744eb6p-6f, 0x1.9615acp-11f};
+    const float d[8] = {0x1p+0f, 0x1.06cefcp+1f, 0x1.ad278ep+0f, 0x1.61293p-1f,
+                        0x1.2f5124p-3f, 0x1.f207a8p-7f, 0x1.1f18ccp-11f, 0x1.20d3f6p-30f};
+    const float e[8] = {0x1.aa1b1cp+2f, 0x1.5daea6p+2f, 0x1.c8ea64p+0f, 0x1.2fad94p-2f,
+                        0x1.b2b412p-6f, 0x1.45c19p-10f, 0x1.c6ec6cp-16f, 0x1.afb74ep-23f};
+    const float f[8] = {0x1p+0f, 0x1.331d34p-1f, 0x1.186eb2p-3f, 0x1.e76f94p-7f,
+                        0x1.9c8bcap-11f, 0x1.35c2c4p-16f, 0x1.31447p-23f, 0x1.269cp-49f};
+    const long long twice = 2ll * (long long)u + 1ll - 4294967296ll;  // 2^33 (U - 1/2), odd
+    const float q = mul(__ll2float_rn(twice), 0x1p-33f);
+    const float aq = q < 0.0f ? -q : q;
+    if (aq <= 0x1.b33334p-2f) {
+        const float r = sub(0x1.71eb86p-3f, mul(q, q));
         return dvd(mul(q, poly7(a, r)), poly7(b, r));
     }
-    const double tail = q < 0.0 ? u : sub(1.0, u);
-    double r = __dsqrt_rn(-det_log(tail));
-    double v;
-    if (r <= 5.0) {
-        r = sub(r, 0x1.999999999999ap+0);
+    const float tail = twice < 0 ? u01(u) : u01(~u);
+    float r = __fsqrt_rn(-det_logf(tail));
+    float v;
+    if (r <= 5.0f) {
+        r = sub(r, 0x1.99999ap+0f);
         v = dvd(poly7(c, r), poly7(d, r));
     } else {
-        r = sub(r, 5.0);
+        r = sub(r, 5.0f);
         v = dvd(poly7(e, r), poly7(f, r));
     }
-    return q < 0.0 ? -v : v;
+    return twice < 0 ? -v : v;
 }
 
 // clip(floor(v + 1/2), lo, hi) for v >= 0 (NaN / inf / huge -> hi)
-__device__ __forceinline__ int64_t round_clip(double v, int64_t lo, int64_t hi)
+__device__ __forceinline__ int64_t round_clip(float v, int64_t lo, int64_t hi)
 {
-    const double y = add(v, 0.5);
-    if (!(y < __ll2double_rn(hi))) return hi;
-    const int64_t t = __double2ll_rz(y);
+    const float y = add(v, 0.5f);
+    if (!(y < __ll2float_rn(hi))) return hi;
+    const int64_t t = __float2ll_rz(y);
     return t < lo ? lo : t;
+}
+
+// floor(num / d) for num >= 0 with recip = floor((2^64 - 1) / d): the estimate is low by at most 2
+__device__ __forceinline__ int64_t div_rate(int64_t num, int64_t d, uint64_t recip)
+{
+    uint64_t q = __umul64hi((uint64_t)num, recip);
+    uint64_t r = (uint64_t)num - q * (uint64_t)d;
+    if (r >= (uint64_t)d) {
+        ++q;
+        r -= (uint64_t)d;
+    }
+    if (r >= (uint64_t)d) ++q;
+    return (int64_t)q;
 }
 
 __device__ __forceinline__ int64_t dwell(const TraceParams& P, uint32_t k0, uint32_t k1, uint32_t sub_id,
                                          int64_t j)
 {
     const U32x4 x = philox((uint32_t)j, sub_id, 1u, 0u, k0, k1);
-    const double g = det_log(u01(x.v[0]));
-    return __double2ll_rz(mul(-g, __ll2double_rn(P.dwell_mean_us)));
+    const float g = det_logf(u01(x.v[0]));
+    return __float2ll_rz(mul(-g, __ll2float_rn(P.dwell_mean_us)));
 }
 
 __global__ void __launch_bounds__(256) trace_kernel(const TraceParams P)
@@ -195,17 +199,17 @@ __global__ void __launch_bounds__(256) trace_kernel(const TraceParams P)
             if (live) {
                 const U32x4 x = philox((uint32_t)k, sub_id, 0u, 0u, k0, k1);
                 const U32x4 y = philox((uint32_t)k, sub_id, 0u, 1u, k0, k1);
-                const double zp = det_ndtri(u01(x.v[0]));
-                p = round_clip(det_exp(add(P.prompt_mu, mul(P.prompt_sigma, zp))), P.prompt_min, P.prompt_max);
+                const float zp = det_ndtrif(x.v[0]);
+                p = round_clip(det_expf(add(P.prompt_mu, mul(P.prompt_sigma, zp))), P.prompt_min, P.prompt_max);
                 const bool is_short = (uint64_t)x.v[1] < P.mix_short_thr;
-                const double mu = is_short ? P.short_mu : P.long_mu;
-                const double sg = is_short ? P.short_sigma : P.long_sigma;
-                const double zo = det_ndtri(u01(x.v[2]));
-                o = round_clip(det_exp(add(mu, mul(sg, zo))), P.out_min, P.out_max);
-                const double zn = det_ndtri(u01(x.v[3]));
-                oh = round_clip(mul(__ll2double_rn(o), det_exp(mul(P.noise_sigma, zn))), P.pred_min, P.pred_max);
+                const float mu = is_short ? P.short_mu : P.long_mu;
+                const float sg = is_short ? P.short_sigma : P.long_sigma;
+                const float zo = det_ndtrif(x.v[2]);
+                o = round_clip(det_expf(add(mu, mul(sg, zo))), P.out_min, P.out_max);
+                const float zn = det_ndtrif(x.v[3]);
+                oh = round_clip(mul(__ll2float_rn(o), det_expf(mul(P.noise_sigma, zn))), P.pred_min, P.pred_max);
                 while (c < P.n_classes - 1 && (uint64_t)y.v[0] >= P.class_thr[c]) ++c;
-                gap = __double2ll_rz(mul(-det_log(u01(y.v[1])), 1e9));
+                gap = __float2ll_rz(mul(-det_logf(u01(y.v[1])), 0x1.dcd65p+29f));
             }
             // inclusive warp scan of the gaps (integers: exact in any order)
             int64_t lam = gap;
@@ -219,13 +223,13 @@ __global__ void __launch_bounds__(256) trace_kernel(const TraceParams P)
 
             int64_t t = 0;
             if (P.arrival_kind == 0) {
-                t = lam / P.rate[0];
+                t = div_rate(lam, P.rate[0], P.rate_recip[0]);
             } else {
                 // walk the intervals until every live lane found the last j with A_j <= lam
                 bool done = !live;
                 for (;;) {
                     if (!done && lam < A_next) {
-                        t = T + (lam - A) / P.rate[j & 1];
+                        t = T + div_rate(lam - A, P.rate[j & 1], P.rate_recip[j & 1]);
                         done = true;
                     }
                     if (__all_sync(0xffffffffu, done)) break;
