@@ -40,6 +40,7 @@ struct __align__(16) Smem {
     int pareto[4][kMaxInst];
     float seg_lo[4][kMaxInst];
     int seg_id[4][kMaxInst];
+    float4 brk[4][2];  // breakpoints 1..7 of each class (seg_lo[s][1..7]), +inf past the last
     int nseg[4];
     unsigned long long bar;
 };
@@ -73,13 +74,25 @@ __device__ __forceinline__ void line_of(const Smem& sm, const ScoreParams& P, in
     m = sig * P.c[1] * P.c[6] * P.c[3] * sm.kap[d];
 }
 
-__device__ __forceinline__ float cost_of(const Smem& sm, const ScoreParams& P, float p, float oh, int s, int d)
+// The request-only part of the cost: own = G + H * kappa_d with
+// G = tau_pre0 + tau_pre p + tau_dec o_hat (1 + rho (p + o_hat) / C) and H = tau_dec rho o_hat,
+// so cost = sigma_s (BK_d + w_s (G + H kappa_d)) + WQA_d.
+struct ReqTerms {
+    float g, h;
+};
+
+__device__ __forceinline__ ReqTerms req_terms(const ScoreParams& P, float p, float oh)
 {
-    const float x2 = fmaf(p + oh, P.c[8], sm.kap[d]);       // post-admission pressure
-    const float x3 = fmaf(P.c[3], x2, 1.0f);                // 1 + rho * press
-    const float own = fmaf(P.c[6] * oh, x3, fmaf(P.c[5], p, P.c[4]));
-    const float y = fmaf(P.c[1], own, sm.bk[d]);
-    return fmaf(P.c[9 + s], y, sm.wqa[d]);
+    const float toh = P.c[6] * oh;                                   // tau_dec o_hat
+    const float press_req = (p + oh) * P.c[8];                       // (p + o_hat) / C
+    const float g = fmaf(toh, fmaf(P.c[3], press_req, 1.0f), fmaf(P.c[5], p, P.c[4]));
+    return ReqTerms{g, toh * P.c[3]};
+}
+
+__device__ __forceinline__ float cost_at(const Smem& sm, const ScoreParams& P, ReqTerms r, int s, int d)
+{
+    const float own = fmaf(r.h, sm.kap[d], r.g);
+    return fmaf(P.c[9 + s], fmaf(P.c[1], own, sm.bk[d]), sm.wqa[d]);
 }
 
 __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, float p, float oh, uint32_t s,
@@ -91,16 +104,145 @@ __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, 
         return;
     }
     const int ns = sm.nseg[s];
-    int lo = 0;
-    int span = ns;
-    while (span > 1) {  // last segment whose left end is <= o_hat
-        const int half = span >> 1;
-        if (sm.seg_lo[s][lo + half] <= oh) lo += half;
-        span -= half;
+    int seg;
+    if (ns <= 8) {  // segments start at 0 and at the sorted breakpoints: count those <= o_hat
+        const float4 b0 = sm.brk[s][0], b1 = sm.brk[s][1];
+        seg = (int)(b0.x <= oh) + (int)(b0.y <= oh) + (int)(b0.z <= oh) + (int)(b0.w <= oh) + (int)(b1.x <= oh) +
+              (int)(b1.y <= oh) + (int)(b1.z <= oh);
+    } else {
+        int lo = 0, span = ns;
+        while (span > 1) {  // last segment whose left end is <= o_hat
+            const int half = span >> 1;
+            if (sm.seg_lo[s][lo + half] <= oh) lo += half;
+            span -= half;
+        }
+        seg = lo;
     }
-    const int d = sm.seg_id[s][lo];
+    const int d = sm.seg_id[s][seg];
     arg = d;
-    cost = cost_of(sm, P, p, oh, (int)s, d);
+    cost = cost_at(sm, P, req_terms(P, p, oh), (int)s, d);
+}
+
+// (intercept, slope, index) lexicographic order of envelope lines
+__device__ __forceinline__ bool line_less(float a, float m, int i, float b, float n, int j)
+{
+    return a < b || (a == b && (m < n || (m == n && i < j)));
+}
+
+// Lower envelope of one class's lines with one warp, for up to 64 lines:
+// a bitonic sort by (intercept, slope, index) across the lanes (two lines per
+// lane), an exclusive prefix minimum of the slopes that keeps the Pareto
+// lines (those whose slope is below every line sorted before them), and the
+// convex-hull stack pass over the survivors by lane 0, which writes the
+// segments' left ends and lines.
+__device__ void warp_envelope(Smem& sm, int s, int n_inst, int lane)
+{
+    float a[2], m[2];
+    int id[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+        const int j = lane + 32 * r;
+        const bool real = j < n_inst;
+        a[r] = real ? sm.la[s][j] : __int_as_float(0x7f800000);
+        m[r] = real ? sm.lm[s][j] : __int_as_float(0x7f800000);
+        id[r] = real ? j : 1 << 20;
+    }
+#pragma unroll
+    for (int k = 2; k <= 64; k <<= 1) {
+#pragma unroll
+        for (int jj = k >> 1; jj > 0; jj >>= 1) {
+            if (jj == 32) {  // partner in the same lane, other slot
+                const bool asc = (lane & k) == 0;  // element index lane has bit 5 clear
+                const bool sw = asc == line_less(a[1], m[1], id[1], a[0], m[0], id[0]);
+                if (sw) {
+                    float t = a[0]; a[0] = a[1]; a[1] = t;
+                    t = m[0]; m[0] = m[1]; m[1] = t;
+                    const int u = id[0]; id[0] = id[1]; id[1] = u;
+                }
+            } else {
+#pragma unroll
+                for (int r = 0; r < 2; ++r) {
+                    const int j = lane + 32 * r;
+                    const float pa = __shfl_xor_sync(0xffffffffu, a[r], jj);
+                    const float pm = __shfl_xor_sync(0xffffffffu, m[r], jj);
+                    const int pi = __shfl_xor_sync(0xffffffffu, id[r], jj);
+                    const bool asc = (j & k) == 0;
+                    const bool lower = (j & jj) == 0;  // this element takes the smaller key when ascending
+                    const bool p_less = line_less(pa, pm, pi, a[r], m[r], id[r]);
+                    if (lower == asc ? p_less : !p_less) {
+                        a[r] = pa;
+                        m[r] = pm;
+                        id[r] = pi;
+                    }
+                }
+            }
+        }
+    }
+    // exclusive prefix minimum of the slopes in sorted order (element j = lane + 32 r)
+    float incl0 = m[0];
+    for (int off = 1; off < 32; off <<= 1) {
+        const float v = __shfl_up_sync(0xffffffffu, incl0, off);
+        if (lane >= off) incl0 = fminf(incl0, v);
+    }
+    const float all0 = __shfl_sync(0xffffffffu, incl0, 31);
+    float excl0 = __shfl_up_sync(0xffffffffu, incl0, 1);
+    if (lane == 0) excl0 = __int_as_float(0x7f800000);
+    float incl1 = m[1];
+    for (int off = 1; off < 32; off <<= 1) {
+        const float v = __shfl_up_sync(0xffffffffu, incl1, off);
+        if (lane >= off) incl1 = fminf(incl1, v);
+    }
+    float excl1 = __shfl_up_sync(0xffffffffu, incl1, 1);
+    excl1 = lane == 0 ? all0 : fminf(excl1, all0);
+    const bool par0 = id[0] < (1 << 20) && m[0] < excl0;
+    const bool par1 = id[1] < (1 << 20) && m[1] < excl1;
+    // compact the Pareto lines, in sorted order, into the segment arrays as scratch
+    const uint32_t b0 = __ballot_sync(0xffffffffu, par0), b1 = __ballot_sync(0xffffffffu, par1);
+    const uint32_t below = (1u << lane) - 1u;
+    if (par0) {
+        const int pos = __popc(b0 & below);
+        sm.lo_tmp[s][pos] = a[0];
+        sm.seg_lo[s][pos] = m[0];
+        sm.valid_tmp[s][pos] = id[0];
+    }
+    if (par1) {
+        const int pos = __popc(b0) + __popc(b1 & below);
+        sm.lo_tmp[s][pos] = a[1];
+        sm.seg_lo[s][pos] = m[1];
+        sm.valid_tmp[s][pos] = id[1];
+    }
+    __syncwarp();
+    if (lane == 0) {  // lower hull: slopes strictly decrease, intercepts strictly increase
+        const int np = __popc(b0) + __popc(b1);
+        int top = 0;  // stack kept in place at the front of the scratch arrays
+        for (int t = 0; t < np; ++t) {
+            const float at = sm.lo_tmp[s][t], mt = sm.seg_lo[s][t];
+            const int it = sm.valid_tmp[s][t];
+            while (top >= 2) {
+                const float a1 = sm.lo_tmp[s][top - 2], m1 = sm.seg_lo[s][top - 2];
+                const float a2 = sm.lo_tmp[s][top - 1], m2 = sm.seg_lo[s][top - 1];
+                // the previous top wins nowhere if the new line meets the one below it no later
+                // (at - a1) / (m1 - mt) <= (a2 - a1) / (m1 - m2), denominators positive
+                if ((at - a1) * (m1 - m2) <= (a2 - a1) * (m1 - mt)) --top;
+                else break;
+            }
+            sm.lo_tmp[s][top] = at;
+            sm.seg_lo[s][top] = mt;
+            sm.valid_tmp[s][top] = it;
+            ++top;
+        }
+        // segment t covers o_hat from the crossing of lines t-1 and t
+        float prev_a = 0.0f, prev_m = 0.0f;
+        for (int t = 0; t < top; ++t) {
+            const float at = sm.lo_tmp[s][t], mt = sm.seg_lo[s][t];
+            const int it = sm.valid_tmp[s][t];
+            sm.seg_lo[s][t] = t == 0 ? 0.0f : (at - prev_a) / (prev_m - mt);
+            sm.seg_id[s][t] = it;
+            prev_a = at;
+            prev_m = mt;
+        }
+        sm.nseg[s] = top;
+    }
 }
 
 template <bool kVec>
@@ -111,7 +253,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     const int tid = threadIdx.x;
     const int n_inst = P.n_inst;
 
-    // first request vector of this thread, in flight while the block builds its envelopes
+    // the first two request vectors of this thread, in flight while the block builds its envelopes
     const int64_t nv = kVec ? (P.n >> 2) : 0;
     const int64_t stride = (int64_t)gridDim.x * kThreads;
     int64_t v = (int64_t)blockIdx.x * kThreads + tid;
@@ -119,12 +261,18 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     const float4* p4 = reinterpret_cast<const float4*>(P.p);
     const float4* o4 = reinterpret_cast<const float4*>(P.oh);
     const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
-    float4 pv = make_float4(0.f, 0.f, 0.f, 0.f), ov = pv;
-    uint32_t cv = 0;
+    float4 pv = make_float4(0.f, 0.f, 0.f, 0.f), ov = pv, pn = pv, on = pv;
+    uint32_t cv = 0, cn = 0;
     if (has) {
         pv = ld_stream(p4 + v);
         ov = ld_stream(o4 + v);
         cv = ld_stream_u32(c4 + v);
+    }
+    bool hn = kVec && v + stride < nv;
+    if (hn) {
+        pn = ld_stream(p4 + v + stride);
+        on = ld_stream(o4 + v + stride);
+        cn = ld_stream_u32(c4 + v + stride);
     }
 
     // ---- stage the instance state: TMA bulk copy when aligned, else plain loads
@@ -191,53 +339,76 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         const int s = idx / n_inst, d = idx - s * n_inst;
         line_of(sm, P, s, d, sm.la[s][d], sm.lm[s][d]);
     }
-    __syncthreads();
-    for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {  // Pareto filter (ties: lowest index survives)
-        const int s = idx / n_inst, d = idx - s * n_inst;
-        const float ad = sm.la[s][d], md = sm.lm[s][d];
-        bool dominated = false;
-        for (int e = 0; e < n_inst; ++e) {
-            const float ae = sm.la[s][e], me = sm.lm[s][e];
-            dominated |= ae <= ad && me <= md && (ae < ad || me < md || e < d);
-        }
-        sm.pareto[s][d] = !dominated;
-    }
-    __syncthreads();
-    for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {  // winning o_hat interval of each surviving line
-        const int s = idx / n_inst, d = idx - s * n_inst;
-        bool valid = false;
-        float lo = 0.0f;
-        if (sm.pareto[s][d]) {
-            const float ad = sm.la[s][d], md = sm.lm[s][d];
-            float hi = __int_as_float(0x7f800000);
-            for (int e = 0; e < n_inst; ++e) {
-                if (e == d || !sm.pareto[s][e]) continue;
-                const float ae = sm.la[s][e], me = sm.lm[s][e];
-                if (me > md) {
-                    lo = fmaxf(lo, (ad - ae) / (me - md));
-                } else if (me < md) {
-                    hi = fminf(hi, (ae - ad) / (md - me));
-                }
-            }
-            valid = lo < hi;
-        }
-        sm.valid_tmp[s][d] = valid;
-        sm.lo_tmp[s][d] = lo;
-    }
     if (tid < 4) sm.nseg[tid] = 0;
     __syncthreads();
-    for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {
-        const int s = idx / n_inst, d = idx - s * n_inst;
-        if (!sm.valid_tmp[s][d]) continue;
-        const float lo = sm.lo_tmp[s][d];
-        int rank = 0;
-        for (int e = 0; e < n_inst; ++e)
-            rank += sm.valid_tmp[s][e] && (sm.lo_tmp[s][e] < lo || (sm.lo_tmp[s][e] == lo && e < d));
-        sm.seg_lo[s][rank] = lo;
-        sm.seg_id[s][rank] = d;
-        atomicAdd(&sm.nseg[s], 1);
+    if (n_inst <= 64) {
+        if (tid < 128) warp_envelope(sm, tid >> 5, n_inst, tid & 31);  // one warp per class
+        __syncthreads();
+    } else {
+        // wider pools: each (class, line) pair is handled by tpp threads that
+        // split its scans over the other lines and combine them with butterfly
+        // shuffles, so all 32 warps of the block share the O(n^2) work
+    int tpp = kThreads / (4 * n_inst);  // threads per pair: a power of two in [1, 32]
+    tpp = tpp >= 32 ? 32 : tpp >= 16 ? 16 : tpp >= 8 ? 8 : tpp >= 4 ? 4 : tpp >= 2 ? 2 : 1;
+    const int pair = tid / tpp, part = tid - pair * tpp;
+    const bool act = pair < 4 * n_inst;
+    const int es = act ? pair / n_inst : 0;
+    const int ed = act ? pair - es * n_inst : 0;
+    const float ad = sm.la[es][ed], md = sm.lm[es][ed];
+    // Pareto filter: a line with a smaller-or-equal intercept and slope (ties: lowest index) hides it
+    bool dominated = false;
+    if (act) {
+#pragma unroll 4
+        for (int e = part; e < n_inst; e += tpp) {
+            const float ae = sm.la[es][e], me = sm.lm[es][e];
+            dominated |= ae <= ad && me <= md && (ae < ad || me < md || e < ed);
+        }
+    }
+    for (int off = 1; off < tpp; off <<= 1) dominated |= __shfl_xor_sync(0xffffffffu, dominated, off, tpp);
+    if (act && part == 0) sm.pareto[es][ed] = !dominated;
+    __syncthreads();
+    // the o_hat interval on which a surviving line wins
+    const bool cand = act && sm.pareto[es][ed];
+    float lo = 0.0f, hi = __int_as_float(0x7f800000);
+    if (cand) {
+#pragma unroll 4
+        for (int e = part; e < n_inst; e += tpp) {
+            if (e == ed || !sm.pareto[es][e]) continue;
+            const float ae = sm.la[es][e], me = sm.lm[es][e];
+            if (me > md) {
+                lo = fmaxf(lo, (ad - ae) / (me - md));
+            } else if (me < md) {
+                hi = fminf(hi, (ae - ad) / (md - me));
+            }
+        }
+    }
+    for (int off = 1; off < tpp; off <<= 1) {
+        lo = fmaxf(lo, __shfl_xor_sync(0xffffffffu, lo, off, tpp));
+        hi = fminf(hi, __shfl_xor_sync(0xffffffffu, hi, off, tpp));
+    }
+    const bool valid = cand && lo < hi;
+    if (act && part == 0) {
+        sm.valid_tmp[es][ed] = valid;
+        sm.lo_tmp[es][ed] = lo;
     }
     __syncthreads();
+    // rank of each winning interval by its left end
+    int rank = 0;
+    if (valid) {
+#pragma unroll 4
+        for (int e = part; e < n_inst; e += tpp) {
+            const float le = sm.lo_tmp[es][e];
+            rank += sm.valid_tmp[es][e] && (le < lo || (le == lo && e < ed));
+        }
+    }
+    for (int off = 1; off < tpp; off <<= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off, tpp);
+    if (valid && part == 0) {
+        sm.seg_lo[es][rank] = lo;
+        sm.seg_id[es][rank] = ed;
+        atomicAdd(&sm.nseg[es], 1);
+    }
+    __syncthreads();
+    }
     if (tid < 4 && sm.nseg[tid] == 0) {  // rounding left no winner (never with finite inputs): brute force line
         int best = 0;
         float bv = 0.0f;
@@ -255,19 +426,26 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     }
     __syncthreads();
 
+    if (tid < 4 * 8) {  // padded breakpoints for the branch-free segment count
+        const int cs = tid >> 3, t = (tid & 7) + 1;
+        float* b = reinterpret_cast<float*>(&sm.brk[cs][0]);
+        b[t - 1] = t < sm.nseg[cs] ? sm.seg_lo[cs][t] : __int_as_float(0x7f800000);
+    }
+    __syncthreads();
+
     // ---- stream the requests (the first vector was loaded before the prologue)
     if (kVec) {
         int4* a4 = reinterpret_cast<int4*>(P.argmin);
         float4* f4 = reinterpret_cast<float4*>(P.cost);
-        while (has) {
-            const int64_t vn = v + stride;
-            const bool hn = vn < nv;
-            float4 pn = make_float4(0.f, 0.f, 0.f, 0.f), on = pn;
-            uint32_t cn = 0;
-            if (hn) {
-                pn = ld_stream(p4 + vn);
-                on = ld_stream(o4 + vn);
-                cn = ld_stream_u32(c4 + vn);
+        while (has) {  // two vectors ahead: v is computed while v + stride and v + 2 stride load
+            const int64_t vf = v + 2 * stride;
+            const bool hf = vf < nv;
+            float4 pf = make_float4(0.f, 0.f, 0.f, 0.f), of = pf;
+            uint32_t cf = 0;
+            if (hf) {
+                pf = ld_stream(p4 + vf);
+                of = ld_stream(o4 + vf);
+                cf = ld_stream_u32(c4 + vf);
             }
             int4 ai;
             float4 fc;
@@ -277,11 +455,15 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
             score_one(sm, P, pv.w, ov.w, cv >> 24, ai.w, fc.w);
             __stcs(a4 + v, ai);
             __stcs(f4 + v, fc);
-            v = vn;
+            v += stride;
             has = hn;
             pv = pn;
             ov = on;
             cv = cn;
+            hn = hf;
+            pn = pf;
+            on = of;
+            cn = cf;
         }
         if (blockIdx.x == 0 && tid < (int)(P.n & 3)) {
             const int64_t i = (nv << 2) + tid;

@@ -39,6 +39,19 @@ constexpr int64_t kBacklogClamp = int64_t(1) << 40;
 constexpr int64_t kPressureClamp = int64_t(1) << 18;
 constexpr int kRecipN = 1024;  // batch sizes with a tabulated reciprocal
 
+// floor((2^64 - 1) / n) for n = 1..kRecipN, for the decode backlog's division
+// by the batch size (built at compile time, read through the read-only path)
+struct RecipTable {
+    uint64_t v[kRecipN + 1];
+};
+constexpr RecipTable make_recip_table()
+{
+    RecipTable t{};
+    for (int i = 1; i <= kRecipN; ++i) t.v[i] = ~0ull / (uint64_t)i;
+    return t;
+}
+__device__ const RecipTable kRecipTable = make_recip_table();
+
 __device__ __forceinline__ uint64_t mix64(uint64_t z)  // splitmix64 output function
 {
     z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
@@ -275,13 +288,9 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // the per-lane event loops, the per-group argmins and the commits are
 // independent across groups.
 template <int G>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32, 4) sim_kernel(const __grid_constant__ SimParams P)
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __grid_constant__ SimParams P)
 {
     constexpr int kRowsPerWarp = 32 / G;
-    // floor((2^64 - 1) / n) for the decode backlog's division by the batch size
-    __shared__ uint64_t recip[kRecipN + 1];
-    for (int i = threadIdx.x; i <= kRecipN; i += blockDim.x) recip[i] = i == 0 ? 0 : ~0ull / (uint64_t)i;
-    __syncthreads();
     const int lane = threadIdx.x & 31;
     const int grp = lane / G;
     const int gl = lane % G;
@@ -393,7 +402,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 4) sim_kernel(const __gri
                                 b = kBacklogClamp;
                             } else {
                                 const uint64_t nd = (uint64_t)(na > 1 ? na : 1);
-                                b = (int64_t)(nd <= (uint64_t)kRecipN ? div_recip(lo, nd, recip[nd]) : lo / nd);
+                                b = (int64_t)(nd <= (uint64_t)kRecipN ? div_recip(lo, nd, __ldg(&kRecipTable.v[nd])) : lo / nd);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
                             int64_t press = (int64_t)div_recip((uint64_t)(s.kv_res + pk + ohk) << 16,
