@@ -144,12 +144,15 @@ def run_reference(args, rank, world):
 
 
 # ---------------------------------------------------------------- GPU arm
+SIM_SOURCES = ("paper_2609_16206_gb300/csrc/sim.cu", "paper_2609_16206_gb300/csrc/ctr_internal.cuh", "include/ctr.h")
+
+
 def _source_hash() -> str:
+    """Hash of the files that define the simulator kernel."""
     h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2609_16206_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode() + f.read())
+    for rel in SIM_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(rel.encode() + f.read())
     return h.hexdigest()[:16]
 
 

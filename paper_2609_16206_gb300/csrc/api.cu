@@ -114,6 +114,7 @@ int ctr_gen_trace(const ctr_trace_cfg* cfg, int32_t n_replicas, int64_t replica_
     p.rate_recip[0] = ~0ull / (uint64_t)cfg->rate_mreq[0];
     p.rate_recip[1] = ~0ull / (uint64_t)cfg->rate_mreq[1];
     p.dwell_mean_us = cfg->dwell_mean_us;
+    p.dwell_mean_f = (float)cfg->dwell_mean_us;
     // the trace is defined in fp32: each parameter is rounded once from the caller's double
     p.prompt_mu = (float)cfg->prompt_mu;
     p.prompt_sigma = (float)cfg->prompt_sigma;

@@ -24,6 +24,7 @@ struct TraceParams {
     int64_t rate[2];
     uint64_t rate_recip[2];     // floor((2^64 - 1) / rate)
     int64_t dwell_mean_us;
+    float dwell_mean_f;         // dwell_mean_us rounded once to fp32
     float prompt_mu, prompt_sigma, short_mu, short_sigma, long_mu, long_sigma, noise_sigma;
     int64_t prompt_min, prompt_max, out_min, out_max, pred_min, pred_max;
     uint64_t mix_short_thr;

@@ -228,6 +228,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                     pos = pos + 1 == P.cap_wait ? 0 : pos + 1;
                 }
             }
+            if (s.w_n == 0) s.w_head = 0;  // an empty ring restarts at its first entry (stays cache-resident)
         }
     }
 }
@@ -376,6 +377,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                             ring_n -= 1;
                             ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
                         }
+                        if (ring_n == 0) ring_head = 0;
                     }
                 }
                 if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;

@@ -49,10 +49,31 @@ __device__ __forceinline__ float sub(float a, float b) { return __fsub_rn(a, b);
 __device__ __forceinline__ float mul(float a, float b) { return __fmul_rn(a, b); }
 __device__ __forceinline__ float dvd(float a, float b) { return __fdiv_rn(a, b); }
 
+// Integer <-> float conversions without the 64-bit conversion instructions
+// (GB300 runs those on its narrow fp64 pipe).  rn_u33(n): n < 2^33 rounded
+// once to fp32 -- the exact sum of two exactly representable parts, rounded by
+// one fp32 addition; trunc_pos(v): the integer part of a non-negative finite
+// float below 2^63, read off its exponent and mantissa.
+__device__ __forceinline__ float rn_u33(uint64_t n)
+{
+    const float hi = __uint2float_rn((uint32_t)(n >> 9));   // < 2^24: exact
+    const float lo = __uint2float_rn((uint32_t)(n & 511u));  // exact
+    return add(mul(hi, 512.0f), lo);
+}
+
+__device__ __forceinline__ int64_t trunc_pos(float v)
+{
+    const uint32_t b = __float_as_uint(v);
+    const int e = (int)((b >> 23) & 0xffu) - 127;  // -0.0 (from ln 1) has e < 0 and gives 0
+    if (e < 0) return 0;
+    const uint64_t mant = (uint64_t)((b & 0x007FFFFFu) | 0x00800000u);
+    return (int64_t)(e >= 23 ? mant << (e - 23) : mant >> (23 - e));
+}
+
 // (u + 1/2) 2^-32 rounded once to fp32; 1 - U is the same of ~u
 __device__ __forceinline__ float u01(uint32_t u)
 {
-    return mul(__ll2float_rn((long long)(2ull * u + 1ull)), 0x1p-33f);
+    return mul(rn_u33(2ull * u + 1ull), 0x1p-33f);
 }
 
 // Natural log of a positive normal x: x = m 2^e with m in (sqrt(1/2), sqrt(2)],
@@ -123,8 +144,9 @@ __device__ float det_ndtrif(uint32_t u)
                         0x1.b2b412p-6f, 0x1.45c19p-10f, 0x1.c6ec6cp-16f, 0x1.afb74ep-23f};
     const float f[8] = {0x1p+0f, 0x1.331d34p-1f, 0x1.186eb2p-3f, 0x1.e76f94p-7f,
                         0x1.9c8bcap-11f, 0x1.35c2c4p-16f, 0x1.31447p-23f, 0x1.269cp-49f};
-    const long long twice = 2ll * (long long)u + 1ll - 4294967296ll;  // 2^33 (U - 1/2), odd
-    const float q = mul(__ll2float_rn(twice), 0x1p-33f);
+    const long long twice = 2ll * (long long)u + 1ll - 4294967296ll;  // 2^33 (U - 1/2), odd, |twice| < 2^32
+    const float mag = __uint2float_rn((uint32_t)(twice < 0 ? -twice : twice));
+    const float q = mul(twice < 0 ? -mag : mag, 0x1p-33f);
     const float aq = q < 0.0f ? -q : q;
     if (aq <= 0x1.b33334p-2f) {
         const float r = sub(0x1.71eb86p-3f, mul(q, q));
@@ -143,12 +165,12 @@ __device__ float det_ndtrif(uint32_t u)
     return twice < 0 ? -v : v;
 }
 
-// clip(floor(v + 1/2), lo, hi) for v >= 0 (NaN / inf / huge -> hi)
+// clip(floor(v + 1/2), lo, hi) for v >= 0 (NaN / inf / huge -> hi); hi <= 2^20
 __device__ __forceinline__ int64_t round_clip(float v, int64_t lo, int64_t hi)
 {
     const float y = add(v, 0.5f);
-    if (!(y < __ll2float_rn(hi))) return hi;
-    const int64_t t = __float2ll_rz(y);
+    if (!(y < __int2float_rn((int)hi))) return hi;
+    const int64_t t = __float2int_rz(y);
     return t < lo ? lo : t;
 }
 
@@ -170,7 +192,7 @@ __device__ __forceinline__ int64_t dwell(const TraceParams& P, uint32_t k0, uint
 {
     const U32x4 x = philox((uint32_t)j, sub_id, 1u, 0u, k0, k1);
     const float g = det_logf(u01(x.v[0]));
-    return __float2ll_rz(mul(-g, __ll2float_rn(P.dwell_mean_us)));
+    return trunc_pos(mul(-g, P.dwell_mean_f));
 }
 
 __global__ void __launch_bounds__(256) trace_kernel(const TraceParams P)
@@ -207,9 +229,9 @@ __global__ void __launch_bounds__(256) trace_kernel(const TraceParams P)
                 const float zo = det_ndtrif(x.v[2]);
                 o = round_clip(det_expf(add(mu, mul(sg, zo))), P.out_min, P.out_max);
                 const float zn = det_ndtrif(x.v[3]);
-                oh = round_clip(mul(__ll2float_rn(o), det_expf(mul(P.noise_sigma, zn))), P.pred_min, P.pred_max);
+                oh = round_clip(mul(__int2float_rn((int)o), det_expf(mul(P.noise_sigma, zn))), P.pred_min, P.pred_max);
                 while (c < P.n_classes - 1 && (uint64_t)y.v[0] >= P.class_thr[c]) ++c;
-                gap = __float2ll_rz(mul(-det_logf(u01(y.v[1])), 0x1.dcd65p+29f));
+                gap = trunc_pos(mul(-det_logf(u01(y.v[1])), 0x1.dcd65p+29f));
             }
             // inclusive warp scan of the gaps (integers: exact in any order)
             int64_t lam = gap;
