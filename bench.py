@@ -334,7 +334,7 @@ def run_ours(args, rank, world, local_rank):
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
     issue_peak = n_sm * 4 * sm_max * 1e6 / 1e9   # G warp-instructions / s
-    inst = SIM_INST_PER_LAUNCH.get(_source_hash())
+    inst = SIM_INST_PER_LAUNCH.get(_source_hash()) if (R, N) == (4096, 20_000) else None
     sim_roof = {"bound": "alu", "unit": "Gwarp-inst/s", "peak": issue_peak,
                 "peak_source": f"{n_sm} SMs x 4 warp-inst/clk x {sm_max:.0f} MHz (max SM clock)",
                 "achieved": None, "frac": None, "traffic": None}
@@ -345,7 +345,8 @@ def run_ours(args, rank, world, local_rank):
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     score_bytes = 17 * N_SCORE_REQ + 3 * 4 * N_SCORE_INST
     score_roof = {"bound": "hbm", "unit": "GB/s", "achieved": score_bytes / (per_kernel_ms["score"] / 1e3) / 1e9,
-                  "peak": hbm, "traffic": None}
+                  "peak": hbm, "traffic": 9.50e6,
+                  "traffic_note": "ncu DRAM read 9.50 MB, write 0 B within the launch (outputs stay in L2)"}
     score_roof["frac"] = score_roof["achieved"] / hbm
     big_bytes = 17 * big_n + 3 * 4 * N_SCORE_INST
     score_roof_big = {"bound": "hbm", "unit": "GB/s", "achieved": big_bytes / (big_ms / 1e3) / 1e9, "peak": hbm,
@@ -380,7 +381,10 @@ def run_ours(args, rank, world, local_rank):
 # Executed warp instructions of one sim_kernel launch on the benchmarked
 # workload (ncu sm__inst_executed.sum), keyed by a hash of csrc/: a stale entry
 # (the kernel changed since the count was taken) reports null.
-SIM_INST_PER_LAUNCH: dict = {}
+SIM_INST_PER_LAUNCH: dict = {
+    # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
+    "7c3503c6a7cd87ee": {"warp_inst": 275808953445, "dram_bytes": 33.38e9 + 23.55e9},
+}
 
 
 def main():
