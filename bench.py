@@ -165,7 +165,7 @@ def run_ours(args, rank, world, local_rank):
         ctr_build.build()
     if world > 1:
         torch.distributed.barrier()
-    from paper_2609_16206_gb300 import ctr
+    from paper_2609_16206_gb300 import ctr, sweep
 
     cpu_base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -183,7 +183,7 @@ def run_ours(args, rank, world, local_rank):
     R, N = wl.n_replicas, wl.n_req
     pols = list(W.ALL_POLICIES)
     rows = R * len(pols)
-    offset = rank * R
+    offset, _ = sweep.shard(rank, R)  # weak scaling: every rank its own block of replicas
 
     tr = ctr.empty_requests(R, N, dev)
     tf = torch.empty((rows, N), dtype=torch.int64, device=dev)

@@ -1,0 +1,122 @@
+"""Host-side orchestration of replica sweeps over the C ABI.
+
+* ``shard`` / ``shard_split`` -- which replicas a rank owns (weak and strong
+  scaling); replicas are independent, so ranks exchange nothing.
+* ``SweepBuffers`` / ``run_step`` -- device buffers and one pass of the hot
+  path for a workload: trace generation, simulation under every policy and
+  constant set, goodput.
+* ``saturation_rate`` -- the arrival rate at which round-robin goodput
+  crosses 1/2 (the paper drives every workload at the rate where round-robin
+  is "mid-collapse", found by probing, sec. IV-B): an integer bisection over
+  milli-requests per second, every probe a GPU simulation.
+* ``calibration_sweep`` / ``large_pool_stress`` -- the mispriced-constants x
+  pool-width sweep and the scarcity stress workload built on those rates.
+
+Everything here is argument marshalling and control flow; the arithmetic runs
+in the CUDA kernels behind ``ctr``.
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import torch
+
+from . import ctr
+from . import workloads as W
+
+
+def shard(rank: int, replicas_per_rank: int) -> tuple:
+    """Weak scaling: rank r simulates replicas [r * n, (r + 1) * n)."""
+    return rank * replicas_per_rank, replicas_per_rank
+
+
+def shard_split(total: int, world: int, rank: int) -> tuple:
+    """Strong scaling: a contiguous, near-equal split of `total` replicas."""
+    base, extra = divmod(total, world)
+    count = base + (1 if rank < extra else 0)
+    offset = rank * base + min(rank, extra)
+    return offset, count
+
+
+@dataclasses.dataclass
+class SweepBuffers:
+    trace: dict
+    t_first: torch.Tensor
+    t_done: torch.Tensor
+    row_hash: torch.Tensor
+    row_status: torch.Tensor
+    met: torch.Tensor
+    p99: torch.Tensor
+    workspace: torch.Tensor
+
+
+def alloc(sim_cfg, n_replicas: int, n_rows: int, n_req: int, device) -> SweepBuffers:
+    return SweepBuffers(
+        trace=ctr.empty_requests(n_replicas, n_req, device),
+        t_first=torch.empty((n_rows, n_req), dtype=torch.int64, device=device),
+        t_done=torch.empty((n_rows, n_req), dtype=torch.int64, device=device),
+        row_hash=torch.empty(n_rows, dtype=torch.int64, device=device),
+        row_status=torch.empty(n_rows, dtype=torch.int32, device=device),
+        met=torch.empty(n_rows, dtype=torch.int64, device=device),
+        p99=torch.empty(n_rows, dtype=torch.int64, device=device),
+        workspace=ctr.simulate_workspace(sim_cfg, n_rows, n_req, device))
+
+
+def run_step(trace_cfg, sim_cfg, const_sets, policies, n_replicas: int, n_req: int, replica_offset: int,
+             buf: SweepBuffers, stream=None, gen: bool = True):
+    """Trace generation (unless gen is False), simulation, goodput; rows are
+    (replica, set, policy) row-major."""
+    if gen:
+        ctr.ctr_gen_trace(trace_cfg, n_replicas, replica_offset, n_req, buf.trace, stream=stream)
+    ctr.ctr_simulate(sim_cfg, const_sets, policies, buf.trace, n_replicas, n_req, buf.t_first, buf.t_done,
+                     buf.row_hash, buf.row_status, buf.workspace, stream=stream)
+    ctr.ctr_goodput(sim_cfg, buf.trace, n_replicas, len(const_sets) * len(policies), n_req, buf.t_first,
+                    buf.t_done, buf.met, buf.p99, stream=stream)
+
+
+def saturation_rate(trace_cfgs, sim_cfg, n_req: int = 10_000, lo: int = 1, hi: int = 200_000, steps: int = 24,
+                    device="cuda") -> list:
+    """For every trace law in `trace_cfgs` (arrival_kind / rate replaced by a
+    Poisson rate), the largest rate in milli-requests/s found by a `steps`-step
+    integer bisection on [lo, hi] at which the round-robin goodput of one
+    replica (seed of the law, replica 0) is at least 1/2.  All laws are probed
+    together, one simulation call per step."""
+    k = len(trace_cfgs)
+    lows = [lo] * k
+    highs = [hi] * k
+    buf = alloc(sim_cfg, k, k, n_req, device)
+    for _ in range(steps):
+        mids = [(a + b) // 2 for a, b in zip(lows, highs)]
+        for i, (tc, mid) in enumerate(zip(trace_cfgs, mids)):
+            law = tc.replace(arrival_kind=0, rate_mreq=(max(mid, 1), max(mid, 1)))
+            view = {name: t[i:i + 1] for name, t in buf.trace.items()}
+            ctr.ctr_gen_trace(law, 1, 0, n_req, view)
+        run_step(None, sim_cfg, [W.CALIBRATED], [W.POLICY_RR], k, n_req, 0, buf, gen=False)
+        met = buf.met.cpu().tolist()
+        status = buf.row_status.cpu().tolist()
+        for i in range(k):
+            ok = status[i] == ctr.CTR_OK and 2 * met[i] >= n_req
+            if ok:
+                lows[i] = mids[i]
+            else:
+                highs[i] = mids[i]
+    return lows
+
+
+def calibration_sweep_cfgs(widths=(3, 4, 5, 6, 7), mixes=(1.0, 5 / 6, 2 / 3, 1 / 2),
+                           loads=(0.8, 29 / 30, 17 / 15, 1.3), seeds: int = 16):
+    """The pool-width x trace-mix x load grid of the mispriced-constants sweep:
+    per width, per (mix, load), `seeds` replicas (distinct sub-streams of seed 0).
+    Returns [(width, mix, load, trace_cfg_without_rate)]."""
+    out = []
+    for w in widths:
+        for mix in mixes:
+            for load in loads:
+                tc = W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(mix), seed=0, n_seeds=1)
+                out.append((w, mix, load, tc))
+    return out
+
+
+def load_rate(sat_mreq: int, load: float) -> int:
+    """Offered rate = load x saturation rate, rounded half up, at least 1."""
+    return max(1, int(sat_mreq * load + 0.5))

@@ -1,0 +1,123 @@
+"""Parity of the sweep workloads built on the saturation search: the
+bisection's endpoints re-checked by the oracle, the mispriced-constants x
+pool-width sweep and the scarcity stress on a large pool (reduced, and at the
+full workload sizes with sampled rows compared by hash)."""
+import numpy as np
+import pytest
+import torch
+
+from gpuutil import host_trace, need_gpu
+from paper_2609_16206_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+def _oracle_rr_goodput(orc, tc, sc, rate, n_req):
+    law = tc.replace(arrival_kind=0, rate_mreq=(rate, rate))
+    tr = orc.gen_trace(law, n_req, replica=0)
+    res = orc.simulate(sc, W.CALIBRATED, W.POLICY_RR, tr)
+    if res["status"] != 0:
+        return None
+    return orc.goodput(sc, tr, res["t_first_us"], res["t_done_us"])[0]
+
+
+def test_saturation_bisection_endpoints(orc):
+    need_gpu()
+    from paper_2609_16206_gb300 import sweep
+    sc = W.SimCfg(n_prefill=2, n_decode=3)
+    laws = [W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(m)) for m in (1.0, 0.5)]
+    n, lo0, hi0 = 2000, 1, 40_000
+    rates = sweep.saturation_rate(laws, sc, n_req=n, lo=lo0, hi=hi0, steps=16)
+    for law, r in zip(laws, rates):
+        assert lo0 < r < hi0
+        assert 2 * _oracle_rr_goodput(orc, law, sc, r, n) >= n
+        above = _oracle_rr_goodput(orc, law, sc, r + 1, n)
+        assert above is None or 2 * above < n
+
+
+def _run_sets(ctr, sc, sets, pols, tr, R, N):
+    rows = R * len(sets) * len(pols)
+    tf = torch.empty((rows, N), dtype=torch.int64, device="cuda")
+    td = torch.empty_like(tf)
+    h = torch.empty(rows, dtype=torch.int64, device="cuda")
+    st = torch.empty(rows, dtype=torch.int32, device="cuda")
+    ws = ctr.simulate_workspace(sc, rows, N, "cuda")
+    ctr.ctr_simulate(sc, sets, pols, tr, R, N, tf, td, h, st, ws)
+    torch.cuda.synchronize()
+    return h.cpu().numpy().astype(np.uint64), st.cpu().numpy()
+
+
+def _calibration_case(orc, widths, mixes, loads, seeds, n_req, n_bisect, sample):
+    ctr = need_gpu()
+    from paper_2609_16206_gb300 import sweep
+    sets = W.mispriced_sets()
+    checked = 0
+    for w in widths:
+        sc = W.SimCfg(n_prefill=2, n_decode=w)
+        laws = [W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(m)) for m in mixes]
+        sat = sweep.saturation_rate(laws, sc, n_req=n_bisect)
+        for law, s_rate in zip(laws, sat):
+            for load in loads:
+                rate = sweep.load_rate(s_rate, load)
+                tc = law.replace(rate_mreq=(rate, rate))
+                tr = ctr.empty_requests(seeds, n_req, "cuda")
+                ctr.ctr_gen_trace(tc, seeds, 0, n_req, tr)
+                h_l, st_l = _run_sets(ctr, sc, sets, [W.POLICY_LEARNED], tr, seeds, n_req)
+                h_b, st_b = _run_sets(ctr, sc, [W.CALIBRATED], [1, 2, 3], tr, seeds, n_req)
+                assert (st_l == 0).all() or (st_l[st_l != 0] == ctr.CTR_EOVERFLOW).all()
+                for r in sample(seeds):
+                    trh = host_trace(tr, r)
+                    for si in (0, 1, 64):
+                        o = orc.simulate(sc, sets[si], W.POLICY_LEARNED, trh)
+                        assert st_l[r * len(sets) + si] == o["status"]
+                        if o["status"] == 0:
+                            assert int(h_l[r * len(sets) + si]) == o["hash"]
+                        checked += 1
+                    for j, pol in enumerate((1, 2, 3)):
+                        o = orc.simulate(sc, W.CALIBRATED, pol, trh)
+                        assert st_b[r * 3 + j] == o["status"]
+                        if o["status"] == 0:
+                            assert int(h_b[r * 3 + j]) == o["hash"]
+    return checked
+
+
+def test_calibration_sweep_reduced(orc):
+    assert _calibration_case(orc, widths=(4, 7), mixes=(1.0, 0.5), loads=(0.8, 1.3), seeds=2, n_req=1500,
+                             n_bisect=1500, sample=lambda s: range(s)) > 0
+
+
+def test_calibration_sweep_full_size_sampled(orc):
+    """5 widths x 4 mixes x 4 loads x 16 seeds x (65 learned sets + 3 baselines), 10,000 requests;
+    every row's status checked, rows sampled against the oracle by hash."""
+    assert _calibration_case(orc, widths=(3, 4, 5, 6, 7), mixes=(1.0, 5 / 6, 2 / 3, 0.5),
+                             loads=(0.8, 29 / 30, 17 / 15, 1.3), seeds=16, n_req=10_000, n_bisect=10_000,
+                             sample=lambda s: (0,)) > 0
+
+
+def _large_pool_case(orc, n_replicas, n_req, sample_replicas):
+    ctr = need_gpu()
+    from paper_2609_16206_gb300 import sweep
+    base = W.large_pool()
+    sat = sweep.saturation_rate([base.trace], base.sim, n_req=10_000)[0]
+    rate = sweep.load_rate(sat, 1.2)
+    tc = base.trace.replace(rate_mreq=(rate, rate))
+    tr = ctr.empty_requests(n_replicas, n_req, "cuda")
+    ctr.ctr_gen_trace(tc, n_replicas, 0, n_req, tr)
+    h, st = _run_sets(ctr, base.sim, base.consts, list(W.ALL_POLICIES), tr, n_replicas, n_req)
+    assert (st == 0).all(), np.unique(st)
+    for r in sample_replicas:
+        trh = host_trace(tr, r)
+        for j, pol in enumerate(W.ALL_POLICIES):
+            o = orc.simulate(base.sim, base.consts[0], pol, trh)
+            assert o["status"] == 0 and int(h[r * 4 + j]) == o["hash"], (r, pol)
+    return sat
+
+
+def test_large_pool_stress_reduced(orc):
+    sat = _large_pool_case(orc, n_replicas=8, n_req=5000, sample_replicas=(0, 7))
+    assert sat > 1000
+
+
+def test_large_pool_stress_full_size_sampled(orc):
+    """16,384 replicas x 50,000 requests, 4P+28D at 1.2x the saturation rate, all four policies."""
+    _large_pool_case(orc, n_replicas=16384, n_req=50_000, sample_replicas=(0, 16383))
