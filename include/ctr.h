@@ -42,8 +42,15 @@ enum ctr_policy {
     CTR_POLICY_LEARNED = 0,          /* marginal-cost argmin, sec. III-A / Algorithm 1 */
     CTR_POLICY_ROUND_ROBIN = 1,      /* request k -> instance k mod N, sec. IV-C */
     CTR_POLICY_LEAST_LOADED = 2,     /* argmin of in-flight count (JSQ), sec. IV-C */
-    CTR_POLICY_LENGTH_HEURISTIC = 3  /* predicted-length threshold heuristic, sec. IV-C */
+    CTR_POLICY_LENGTH_HEURISTIC = 3, /* predicted-length threshold heuristic, sec. IV-C */
+    CTR_POLICY_LEARNED_P2 = 4        /* marginal cost over two sampled candidates per pool, sec. V-D / VI */
 };
+
+/* Feature ablation (sec. V-F): bits of ctr_cost_consts.ablate.  A removed
+ * feature takes its neutral value in the learned cost. */
+#define CTR_ABLATE_PREDICTED_LENGTH 1u /* o_hat := 0 (no own decode work, pressure without it) */
+#define CTR_ABLATE_PRESSURE 2u         /* P := 0 */
+#define CTR_ABLATE_SLO 4u              /* sigma := 1.0 (256) for every class */
 
 enum ctr_workspace_kind { CTR_WS_SIMULATE = 0 };
 
@@ -114,13 +121,18 @@ typedef struct ctr_sim_cfg {
  *   T2    = own + floor(floor(own * P / 2^16) * rho / 2^8)
  *   cost  = (w_b * min(B_d, 2^40) + w_s * T2) * sigma[class] + w_q * queue * 2^16
  * Prefill cost: (w_b * B_p + w_s * (tau_pre0 + p * tau_pre)) * sigma[class] + w_q * queue * 2^16,
- * with backlog B_p = max(0, busy_until - t) and B_d = floor(R_d * step_d / max(1, n_d)). */
+ * with backlog B_p = max(0, busy_until - t) and B_d = floor(R_d * step_d / max(1, n_d)).
+ * CTR_POLICY_LEARNED_P2 prices only two candidates per pool: Philox4x32-10
+ * with key (0x243F6A88, 0x85A308D3) and counter (k, t lo, t hi, 0x5032) gives
+ * u0..u3; a pool of n offers c0 = floor(u n / 2^32) and
+ * c1 = (c0 + 1 + floor(u' (n - 1) / 2^32)) mod n (decode (u0, u1), prefill
+ * (u2, u3)), and the cheaper one wins (ties to the lower index). */
 typedef struct ctr_cost_consts {
     int64_t tau_pre0_us, tau_pre_us, tau_dec_us; /* 0..2^20 */
     int64_t w_q_us;                              /* 0..2^20, us per in-flight request */
     int32_t w_b_q8, w_s_q8, rho_q8;              /* 0..1023 */
     int32_t sigma_q8[4];                         /* 0..1023 */
-    int32_t reserved0;
+    uint32_t ablate;                             /* CTR_ABLATE_* bits, 0 = every feature */
 } ctr_cost_consts;
 
 /* ctr_gen_trace -- synthetic request trace (Table 1 length profiles as
@@ -161,7 +173,7 @@ size_t ctr_workspace_bytes(int32_t which, const ctr_sim_cfg* cfg /* host */, int
  *   row = (replica * n_const_sets + set) * n_policies + policy_index.
  * Replica r reads trace[r * n_req + k]; outputs are [row * n_req + k].
  * consts: n_const_sets host structs (1..CTR_MAX_CONST_SETS); policy_ids:
- * n_policies host ints (1..4), values of enum ctr_policy.
+ * n_policies host ints (1..5 of them), values of enum ctr_policy.
  * Outputs: i_pre / i_dec (optional, NULL ok) chosen prefill / decode instance;
  * t_first_us (end of the first decode step) and t_done_us (required);
  * row_hash the order-independent 64-bit checksum of each row's routing and

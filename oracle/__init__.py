@@ -70,7 +70,7 @@ class _SimCfg(C.Structure):
 class _Consts(C.Structure):
     _fields_ = [("tau_pre0", C.c_int64), ("tau_pre", C.c_int64), ("tau_dec", C.c_int64), ("w_q", C.c_int64),
                 ("w_b_q8", C.c_int64), ("w_s_q8", C.c_int64), ("rho_q8", C.c_int64),
-                ("sigma_q8", C.c_int64 * 4)]
+                ("sigma_q8", C.c_int64 * 4), ("ablate", C.c_int64)]
 
 
 class Stats(C.Structure):
@@ -170,6 +170,7 @@ def _consts(cc) -> _Consts:
     sig = list(cc.sigma_q8) + [256] * (4 - len(cc.sigma_q8))
     for i in range(4):
         s.sigma_q8[i] = int(sig[i])
+    s.ablate = int(getattr(cc, "ablate", 0))
     return s
 
 

@@ -325,6 +325,7 @@ typedef struct {
 typedef struct {
     int64_t tau_pre0, tau_pre, tau_dec, w_q;
     int64_t w_b_q8, w_s_q8, rho_q8, sigma_q8[4];
+    int64_t ablate; /* bit 0: predicted length, bit 1: KV pressure, bit 2: SLO class (sec. V-F) */
 } orc_consts;
 
 typedef struct {
@@ -334,7 +335,7 @@ typedef struct {
     int64_t events;                        /* heap events processed */
 } orc_stats;
 
-enum { POL_LEARNED = 0, POL_RR = 1, POL_JSQ = 2, POL_HEUR = 3 };
+enum { POL_LEARNED = 0, POL_RR = 1, POL_JSQ = 2, POL_HEUR = 3, POL_LEARNED_P2 = 4 };
 enum { EV_STEP_END = 0, EV_PREFILL_END = 1, EV_KV_READY = 2 };
 enum { ST_NONE = 0, ST_PENDING = 1, ST_WAITING = 2, ST_ACTIVE = 3, ST_DONE = 4 };
 
@@ -560,6 +561,38 @@ static int64_t decode_backlog(int64_t remaining, int64_t step, int64_t n_active)
     return b < B_CLAMP ? b : B_CLAMP;
 }
 
+/* Power-of-two candidates [reading: the paper names the sampled variant only].
+ * Philox4x32-10 with key (0x243F6A88, 0x85A308D3) and counter
+ * (k, t lo, t hi, 0x5032) gives words u0..u3; a pool of n instances offers
+ * c0 = floor(u * n / 2^32) and c1 = (c0 + 1 + floor(u' (n - 1) / 2^32)) mod n
+ * (distinct when n > 1), decode from (u0, u1), prefill from (u2, u3). */
+static void p2_words(int64_t k, int64_t t, uint32_t out[4])
+{
+    uint32_t ctr[4] = {(uint32_t)k, (uint32_t)t, (uint32_t)((uint64_t)t >> 32), 0x5032u};
+    uint32_t key[2] = {0x243F6A88u, 0x85A308D3u};
+    orc_philox4x32_10(ctr, key, out);
+}
+
+static void p2_pair(uint32_t u, uint32_t v, int64_t n, int64_t c[2])
+{
+    c[0] = (int64_t)(((uint64_t)u * (uint64_t)n) >> 32);
+    c[1] = n > 1 ? (c[0] + 1 + (int64_t)(((uint64_t)v * (uint64_t)(n - 1)) >> 32)) % n : c[0];
+}
+
+static void p2_candidates_dec(int64_t k, int64_t t, int64_t nd, int64_t c[2])
+{
+    uint32_t w[4];
+    p2_words(k, t, w);
+    p2_pair(w[0], w[1], nd, c);
+}
+
+static void p2_candidates(int64_t k, int64_t t, int64_t np, int64_t c[2])
+{
+    uint32_t w[4];
+    p2_words(k, t, w);
+    p2_pair(w[2], w[3], np, c);
+}
+
 /* Route request k at time t (Algorithm 1) and commit it. */
 static int route(sim_t* s, int64_t k, int64_t t)
 {
@@ -574,39 +607,53 @@ static int route(sim_t* s, int64_t k, int64_t t)
         ip = k % np;
         id = k % nd;
     } else {
+        int learned = s->policy == POL_LEARNED || s->policy == POL_LEARNED_P2;
+        /* feature ablation (sec. V-F): a removed feature takes its neutral value */
+        int64_t oh_f = (cc->ablate & 1) ? 0 : ohk;
+        int64_t sig = (cc->ablate & 4) ? 256 : cc->sigma_q8[ck];
         for (int64_t i = 0; i < np; ++i) {
             int64_t q = s->inflight[i];
-            if (s->policy == POL_LEARNED) {
+            if (learned) {
                 int64_t b = s->busy[i] - t;
                 if (b < 0) b = 0;
                 if (b > B_CLAMP) b = B_CLAMP;
                 int64_t own = cc->tau_pre0 + pk * cc->tau_pre;
                 int64_t load = cc->w_b_q8 * b + cc->w_s_q8 * own;
-                cost_p[i] = load * cc->sigma_q8[ck] + cc->w_q * q * 65536;
+                cost_p[i] = load * sig + cc->w_q * q * 65536;
             } else {
                 cost_p[i] = q; /* JSQ and the heuristic place prefill by queue length */
             }
         }
-        ip = argmin_lowest(cost_p, np);
         for (int64_t d = 0; d < nd; ++d) {
             int64_t q = s->n_committed[d];
-            if (s->policy == POL_LEARNED) {
+            if (learned) {
                 int64_t na = dec_active(s, d);
                 int64_t res = dec_resident(s, d);
                 int64_t b = decode_backlog(dec_remaining(s, d), step_time(cfg, na, res), na);
-                int64_t press = ((res + pk + ohk) * 65536) / cfg->kv_cap;
+                int64_t press = ((res + pk + oh_f) * 65536) / cfg->kv_cap;
                 if (press > P_CLAMP) press = P_CLAMP;
-                int64_t own = ohk * cc->tau_dec;
+                if (cc->ablate & 2) press = 0;
+                int64_t own = oh_f * cc->tau_dec;
                 int64_t priced = own + (((own * press) >> 16) * cc->rho_q8 >> 8);
                 int64_t load = cc->w_b_q8 * b + cc->w_s_q8 * priced;
-                cost_d[d] = load * cc->sigma_q8[ck] + cc->w_q * q * 65536;
+                cost_d[d] = load * sig + cc->w_q * q * 65536;
             } else if (s->policy == POL_HEUR && ohk >= cfg->heur_thresh) {
                 cost_d[d] = dec_pred_sum(s, d);
             } else {
                 cost_d[d] = q;
             }
         }
-        id = argmin_lowest(cost_d, nd);
+        if (s->policy == POL_LEARNED_P2) {
+            /* power-of-two choices (sec. V-D, VI): only two sampled candidates per pool are priced */
+            int64_t cp[2], cd[2];
+            p2_candidates(k, t, np, cp);
+            p2_candidates_dec(k, t, nd, cd);
+            ip = cost_p[cp[1]] < cost_p[cp[0]] || (cost_p[cp[1]] == cost_p[cp[0]] && cp[1] < cp[0]) ? cp[1] : cp[0];
+            id = cost_d[cd[1]] < cost_d[cd[0]] || (cost_d[cd[1]] == cost_d[cd[0]] && cd[1] < cd[0]) ? cd[1] : cd[0];
+        } else {
+            ip = argmin_lowest(cost_p, np);
+            id = argmin_lowest(cost_d, nd);
+        }
     }
 
     int64_t start = s->busy[ip] > t ? s->busy[ip] : t;
@@ -657,7 +704,8 @@ static int validate_cfg(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t po
     if (cfg->kv_cap < 1 || cfg->kv_cap > 2147483647LL) return ORC_EINVAL;
     if (cfg->dec_kv_div < 1 || cfg->pre_base < 1 || cfg->dec_base < 1) return ORC_EINVAL;
     if (cfg->n_classes < 1 || cfg->n_classes > 4) return ORC_EINVAL;
-    if (policy < 0 || policy > 3) return ORC_EINVAL;
+    if (policy < 0 || policy > 4) return ORC_EINVAL;
+    if (cc->ablate < 0 || cc->ablate > 7) return ORC_EINVAL;
     if (cc->w_b_q8 < 0 || cc->w_b_q8 > 1023 || cc->w_s_q8 < 0 || cc->w_s_q8 > 1023) return ORC_EINVAL;
     if (cc->rho_q8 < 0 || cc->rho_q8 > 1023) return ORC_EINVAL;
     for (int i = 0; i < 4; ++i)

@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 1;
+constexpr int kAbiVersion = 2;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -53,6 +53,7 @@ bool valid_consts(const ctr_cost_consts& k)
     if (!in_range(k.w_b_q8, 0, 1023) || !in_range(k.w_s_q8, 0, 1023) || !in_range(k.rho_q8, 0, 1023)) return false;
     for (int i = 0; i < 4; ++i)
         if (!in_range(k.sigma_q8[i], 0, 1023)) return false;
+    if (k.ablate > 7u) return false;
     return true;
 }
 
@@ -185,12 +186,12 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
                  int32_t* row_status, void* workspace, size_t workspace_bytes, void* stream)
 {
     if (!valid_sim_cfg(cfg) || !consts || !policy_ids) return CTR_EINVAL;
-    if (!in_range(n_const_sets, 1, CTR_MAX_CONST_SETS) || !in_range(n_policies, 1, 4)) return CTR_EINVAL;
+    if (!in_range(n_const_sets, 1, CTR_MAX_CONST_SETS) || !in_range(n_policies, 1, 5)) return CTR_EINVAL;
     if (n_replicas < 0 || !in_range(n_req, 0, CTR_MAX_REQUESTS)) return CTR_EINVAL;
     for (int i = 0; i < n_const_sets; ++i)
         if (!valid_consts(consts[i])) return CTR_EINVAL;
     for (int i = 0; i < n_policies; ++i)
-        if (!in_range(policy_ids[i], 0, 3)) return CTR_EINVAL;
+        if (!in_range(policy_ids[i], 0, 4)) return CTR_EINVAL;
     const int64_t n_rows = (int64_t)n_replicas * n_const_sets * n_policies;
     if (n_rows >= (1LL << 31)) return CTR_EINVAL;
     if (n_rows == 0) return CTR_OK;
@@ -249,6 +250,7 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
         d.w_s = k.w_s_q8;
         d.rho = k.rho_q8;
         for (int c = 0; c < 4; ++c) d.sigma[c] = k.sigma_q8[c];
+        d.ablate = k.ablate;
     }
 
     p.slot_bytes = sim_slot_bytes(*cfg, &p.off_act, &p.off_wait, &p.cap_pr);

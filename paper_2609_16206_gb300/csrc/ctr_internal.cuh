@@ -15,6 +15,29 @@ constexpr int64_t kArrivalLimit = int64_t(1) << 39;
 constexpr int kKeyBits = 23;                        // request index bits in packed heap keys
 constexpr uint64_t kKeyMask = (uint64_t(1) << kKeyBits) - 1;
 
+// Philox4x32-10 (Salmon et al., SC'11): ten rounds of two 32x32 -> 64 products,
+// the key bumped by the Weyl constants between rounds.
+struct Philox4 {
+    uint32_t v[4];
+};
+__device__ __forceinline__ Philox4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3, uint32_t k0,
+                                                 uint32_t k1)
+{
+#pragma unroll
+    for (int round = 0; round < 10; ++round) {
+        const uint32_t hi0 = __umulhi(0xD2511F53u, c0), lo0 = 0xD2511F53u * c0;
+        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2), lo1 = 0xCD9E8D57u * c2;
+        const uint32_t n0 = hi1 ^ c1 ^ k0, n2 = hi0 ^ c3 ^ k1;
+        c0 = n0;
+        c1 = lo1;
+        c2 = n2;
+        c3 = lo0;
+        k0 += 0x9E3779B9u;  // the bump after the last round is never used
+        k1 += 0xBB67AE85u;
+    }
+    return Philox4{{c0, c1, c2, c3}};
+}
+
 // ---------------------------------------------------------------- trace
 struct TraceParams {
     uint64_t seed;
@@ -38,7 +61,7 @@ cudaError_t launch_trace(const TraceParams& p, cudaStream_t stream);
 struct ConstsDev {
     int64_t tau_pre0, tau_pre, tau_dec, w_q;
     int32_t w_b, w_s, rho, sigma[4];
-    int32_t pad;
+    uint32_t ablate;
 };
 
 struct SimParams {
@@ -53,7 +76,7 @@ struct SimParams {
     int64_t max_steps;
     int32_t cap_pend, cap_wait, cap_act, cap_ring;
     int32_t n_sets, n_pols;
-    int32_t pols[4];
+    int32_t pols[8];
     int64_t n_req, n_rows;
     // per-slot workspace: interleaved [entry][lane] arrays
     unsigned char* ws;

@@ -385,16 +385,20 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                 // 2. price the candidates and take the argmin of each pool
                 uint64_t cost = kEmpty;
                 if (live && pol != CTR_POLICY_ROUND_ROBIN) {
+                    const bool learned = pol == CTR_POLICY_LEARNED || pol == CTR_POLICY_LEARNED_P2;
+                    // feature ablation (sec. V-F): a removed feature takes its neutral value
+                    const int64_t oh_f = (cc.ablate & CTR_ABLATE_PREDICTED_LENGTH) ? 0 : ohk;
+                    const int64_t sig = (cc.ablate & CTR_ABLATE_SLO) ? 256 : cc.sigma[ck];
                     if (is_pre) {
-                        if (pol == CTR_POLICY_LEARNED) {
+                        if (learned) {
                             const int64_t b = busy > T ? busy - T : 0;
                             const int64_t load = cc.w_b * b + cc.w_s * (cc.tau_pre0 + pk * cc.tau_pre);
-                            cost = (uint64_t)(load * cc.sigma[ck] + cc.w_q * (int64_t)ring_n * 65536);
+                            cost = (uint64_t)(load * sig + cc.w_q * (int64_t)ring_n * 65536);
                         } else {
                             cost = (uint64_t)ring_n;
                         }
                     } else if (is_dec) {
-                        if (pol == CTR_POLICY_LEARNED) {
+                        if (learned) {
                             const int64_t na = s.n_act;
                             const int64_t step = P.dec_base + P.dec_seq * na + kv_term(s.kv_res, P);
                             const uint64_t hi = __umul64hi((uint64_t)s.R, (uint64_t)step);
@@ -404,21 +408,38 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                                 b = kBacklogClamp;
                             } else {
                                 const uint64_t nd = (uint64_t)(na > 1 ? na : 1);
-                                b = (int64_t)(nd <= (uint64_t)kRecipN ? div_recip(lo, nd, __ldg(&kRecipTable.v[nd])) : lo / nd);
+                                b = (int64_t)(nd <= (uint64_t)kRecipN ? div_recip(lo, nd, __ldg(&kRecipTable.v[nd]))
+                                                                      : lo / nd);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            int64_t press = (int64_t)div_recip((uint64_t)(s.kv_res + pk + ohk) << 16,
+                            int64_t press = (int64_t)div_recip((uint64_t)(s.kv_res + pk + oh_f) << 16,
                                                                (uint64_t)P.kv_cap, P.kv_cap_recip);
                             if (press > kPressureClamp) press = kPressureClamp;
-                            const int64_t own = ohk * cc.tau_dec;
+                            if (cc.ablate & CTR_ABLATE_PRESSURE) press = 0;
+                            const int64_t own = oh_f * cc.tau_dec;
                             const int64_t priced = own + ((((own * press) >> 16) * cc.rho) >> 8);
                             const int64_t load = cc.w_b * b + cc.w_s * priced;
-                            cost = (uint64_t)(load * cc.sigma[ck] + cc.w_q * (int64_t)s.q * 65536);
+                            cost = (uint64_t)(load * sig + cc.w_q * (int64_t)s.q * 65536);
                         } else if (pol == CTR_POLICY_LENGTH_HEURISTIC && ohk >= P.heur_thresh) {
                             cost = (uint64_t)s.ohat;
                         } else {
                             cost = (uint64_t)s.q;
                         }
+                    }
+                    if (pol == CTR_POLICY_LEARNED_P2 && (is_pre || is_dec)) {
+                        // power of two choices: only two sampled candidates per pool are priced
+                        const Philox4 u = philox4x32_10((uint32_t)k, (uint32_t)T, (uint32_t)((uint64_t)T >> 32),
+                                                        0x5032u, 0x243F6A88u, 0x85A308D3u);
+                        const uint32_t n_pool = is_pre ? (uint32_t)P.n_pre : (uint32_t)P.n_dec;
+                        const uint32_t a0 = is_pre ? u.v[2] : u.v[0], a1 = is_pre ? u.v[3] : u.v[1];
+                        const uint32_t c0 = (uint32_t)(((uint64_t)a0 * n_pool) >> 32);
+                        uint32_t c1 = c0;
+                        if (n_pool > 1) {
+                            c1 = c0 + 1 + (uint32_t)(((uint64_t)a1 * (n_pool - 1)) >> 32);
+                            if (c1 >= n_pool) c1 -= n_pool;
+                        }
+                        const uint32_t me = is_pre ? (uint32_t)gl : (uint32_t)(gl - P.n_pre);
+                        if (me != c0 && me != c1) cost = kEmpty;
                     }
                 }
                 const int amin_p = group_argmin<G>(is_pre ? cost : kEmpty, gl);

@@ -20,27 +20,11 @@
 namespace ctr {
 namespace {
 
-// ------------------------------------------------------------- Philox4x32-10
-struct U32x4 {
-    uint32_t v[4];
-};
-
+using U32x4 = Philox4;
 __device__ __forceinline__ U32x4 philox(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3, uint32_t k0,
                                         uint32_t k1)
 {
-#pragma unroll
-    for (int round = 0; round < 10; ++round) {
-        const uint32_t hi0 = __umulhi(0xD2511F53u, c0), lo0 = 0xD2511F53u * c0;
-        const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2), lo1 = 0xCD9E8D57u * c2;
-        const uint32_t n0 = hi1 ^ c1 ^ k0, n2 = hi0 ^ c3 ^ k1;
-        c0 = n0;
-        c1 = lo1;
-        c2 = n2;
-        c3 = lo0;
-        k0 += 0x9E3779B9u;  // the bump after the last round is never used
-        k1 += 0xBB67AE85u;
-    }
-    return U32x4{{c0, c1, c2, c3}};
+    return philox4x32_10(c0, c1, c2, c3, k0, k1);
 }
 
 // ------------------------------------------------------------- fp32 helpers

@@ -66,7 +66,7 @@ class CtrSimCfg(C.Structure):
 class CtrCostConsts(C.Structure):
     _fields_ = [("tau_pre0_us", C.c_int64), ("tau_pre_us", C.c_int64), ("tau_dec_us", C.c_int64),
                 ("w_q_us", C.c_int64), ("w_b_q8", C.c_int32), ("w_s_q8", C.c_int32), ("rho_q8", C.c_int32),
-                ("sigma_q8", C.c_int32 * 4), ("reserved0", C.c_int32)]
+                ("sigma_q8", C.c_int32 * 4), ("ablate", C.c_uint32)]
 
 
 _lock = threading.Lock()
@@ -181,6 +181,7 @@ def consts_array(sets):
         sig = list(cc.sigma_q8) + [256] * (4 - len(cc.sigma_q8))
         for c in range(4):
             a.sigma_q8[c] = int(sig[c])
+        a.ablate = int(getattr(cc, "ablate", 0))
     return arr
 
 

@@ -24,9 +24,10 @@ LN_128 = float.fromhex("0x1.3687a9f1af2b1p+2")
 LN_512 = float.fromhex("0x1.8f40b5ed9812dp+2")
 LN_1024 = float.fromhex("0x1.bb9d3beb8c86bp+2")
 
-POLICY_LEARNED, POLICY_RR, POLICY_JSQ, POLICY_HEURISTIC = 0, 1, 2, 3
+POLICY_LEARNED, POLICY_RR, POLICY_JSQ, POLICY_HEURISTIC, POLICY_LEARNED_P2 = 0, 1, 2, 3, 4
 POLICY_NAMES = {POLICY_LEARNED: "learned", POLICY_RR: "round_robin", POLICY_JSQ: "least_loaded",
-                POLICY_HEURISTIC: "length_heuristic"}
+                POLICY_HEURISTIC: "length_heuristic", POLICY_LEARNED_P2: "learned_power_of_two"}
+ABLATE_PREDICTED_LENGTH, ABLATE_PRESSURE, ABLATE_SLO = 1, 2, 4
 ALL_POLICIES = (POLICY_LEARNED, POLICY_RR, POLICY_JSQ, POLICY_HEURISTIC)
 
 
@@ -101,6 +102,7 @@ class CostConsts:
     w_s_q8: int = 256
     rho_q8: int = 256
     sigma_q8: tuple = (512, 256, 256, 256)
+    ablate: int = 0                  # ABLATE_* bits: features replaced by their neutral value
 
     def replace(self, **kw) -> "CostConsts":
         return dataclasses.replace(self, **kw)

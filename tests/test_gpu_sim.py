@@ -172,7 +172,8 @@ def test_host_validation_rejects(orc):
     for sc, sets, pols in ((wl.sim.replace(n_prefill=0), [W.CALIBRATED], [0]),
                            (wl.sim.replace(n_prefill=20, n_decode=13), [W.CALIBRATED], [0]),
                            (wl.sim, [W.CALIBRATED.replace(w_b_q8=1024)], [0]),
-                           (wl.sim, [W.CALIBRATED], [4]),
+                           (wl.sim, [W.CALIBRATED], [5]),
+                           (wl.sim, [W.CALIBRATED.replace(ablate=8)], [0]),
                            (wl.sim, [W.CALIBRATED], []),
                            (wl.sim.replace(cap_active=0), [W.CALIBRATED], [0])):
         with pytest.raises(Exception):
@@ -202,3 +203,26 @@ def test_full_size_sweep_sampled(orc):
         for j, pol in enumerate(W.ALL_POLICIES):
             o = orc.simulate(wl.sim, W.CALIBRATED, pol, trh)
             assert o["status"] == 0 and int(hh[r * 4 + j]) == o["hash"], (r, pol)
+
+
+@pytest.mark.parametrize("ablate", [1, 2, 4, 7])
+def test_feature_ablation(orc, ablate):
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    R, N = 6, 2000
+    tr = gen(ctr, wl.trace, R, N)
+    cc = W.CALIBRATED.replace(ablate=ablate)
+    res = simulate(ctr, wl.sim, [cc], [W.POLICY_LEARNED, W.POLICY_LEARNED_P2], tr, R, N)
+    _check_rows(orc, wl.sim, [cc], [W.POLICY_LEARNED, W.POLICY_LEARNED_P2], [host_trace(tr, r) for r in range(R)],
+                res, N)
+
+
+@pytest.mark.parametrize("wl", [W.replica_sweep(), W.large_pool(rate_mreq=34_000), W.single_replica()],
+                         ids=["2p6d", "4p28d", "1p3d"])
+def test_power_of_two_router(orc, wl):
+    ctr = need_gpu()
+    R, N = 4, 2500
+    tr = gen(ctr, wl.trace, R, N)
+    pols = [W.POLICY_LEARNED_P2, W.POLICY_LEARNED, W.POLICY_RR]
+    res = simulate(ctr, wl.sim, [wl.consts[0]], pols, tr, R, N)
+    _check_rows(orc, wl.sim, [wl.consts[0]], pols, [host_trace(tr, r) for r in range(R)], res, N)

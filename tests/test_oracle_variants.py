@@ -1,0 +1,88 @@
+"""Pins for the router variants the paper names (sec. V-D power of two
+choices, sec. V-F feature ablation): cases that reduce to the full router or to
+constants, the documented candidate sampling, and invariance to an ablated
+feature."""
+import numpy as np
+import pytest
+
+from paper_2609_16206_gb300 import workloads as W
+
+
+def _p2_pair(orc, k, t, n_pool, pool):
+    w = orc.philox4x32_10([k & 0xFFFFFFFF, t & 0xFFFFFFFF, (t >> 32) & 0xFFFFFFFF, 0x5032], [0x243F6A88, 0x85A308D3])
+    u, v = (int(w[0]), int(w[1])) if pool == "dec" else (int(w[2]), int(w[3]))
+    c0 = (u * n_pool) >> 32
+    c1 = (c0 + 1 + ((v * (n_pool - 1)) >> 32)) % n_pool if n_pool > 1 else c0
+    return {c0, c1}
+
+
+def test_power_of_two_on_two_instance_pools_is_the_full_argmin(orc):
+    sc = W.SimCfg(n_prefill=2, n_decode=2)
+    tr = orc.gen_trace(W.TraceCfg(rate_mreq=(6000, 6000)), 2000)
+    a = orc.simulate(sc, W.CALIBRATED, W.POLICY_LEARNED, tr)
+    b = orc.simulate(sc, W.CALIBRATED, W.POLICY_LEARNED_P2, tr)
+    assert a["status"] == b["status"] == 0
+    for key in ("i_pre", "i_dec", "t_first_us", "t_done_us"):
+        assert np.array_equal(a[key], b[key])
+
+
+def test_power_of_two_picks_from_its_sampled_pair(orc):
+    wl = W.replica_sweep()
+    tr = orc.gen_trace(wl.trace, 1500, replica=5)
+    res = orc.simulate(wl.sim, W.CALIBRATED, W.POLICY_LEARNED_P2, tr)
+    assert res["status"] == 0
+    full = orc.simulate(wl.sim, W.CALIBRATED, W.POLICY_LEARNED, tr)
+    for k in range(tr["arrival_us"].size):
+        t = int(tr["arrival_us"][k])
+        assert int(res["i_dec"][k]) in _p2_pair(orc, k, t, wl.sim.n_decode, "dec")
+        assert int(res["i_pre"][k]) in _p2_pair(orc, k, t, wl.sim.n_prefill, "pre")
+    assert not np.array_equal(res["i_dec"], full["i_dec"])   # six decode instances: sampling changes routes
+    counts = np.bincount(res["i_dec"], minlength=6)
+    assert counts.min() > 100                                  # every instance gets sampled and used
+
+
+def test_power_of_two_single_instance_pools(orc):
+    sc = W.SimCfg(n_prefill=1, n_decode=1)
+    tr = orc.gen_trace(W.TraceCfg(rate_mreq=(1500, 1500)), 800)
+    a = orc.simulate(sc, W.CALIBRATED, W.POLICY_RR, tr)
+    b = orc.simulate(sc, W.CALIBRATED, W.POLICY_LEARNED_P2, tr)
+    assert a["hash"] == b["hash"]
+
+
+def test_ablate_slo_equals_flat_sigma(orc):
+    wl = W.replica_sweep()
+    tr = orc.gen_trace(wl.trace, 2000, replica=1)
+    a = orc.simulate(wl.sim, W.CALIBRATED.replace(ablate=W.ABLATE_SLO), W.POLICY_LEARNED, tr)
+    b = orc.simulate(wl.sim, W.CALIBRATED.replace(sigma_q8=(256, 256, 256, 256)), W.POLICY_LEARNED, tr)
+    c = orc.simulate(wl.sim, W.CALIBRATED, W.POLICY_LEARNED, tr)
+    assert a["hash"] == b["hash"] and a["hash"] != c["hash"]
+
+
+def test_ablate_pressure_equals_zero_rho(orc):
+    wl = W.replica_sweep()
+    tr = orc.gen_trace(wl.trace, 2000, replica=2)
+    a = orc.simulate(wl.sim, W.CALIBRATED.replace(ablate=W.ABLATE_PRESSURE), W.POLICY_LEARNED, tr)
+    b = orc.simulate(wl.sim, W.CALIBRATED.replace(rho_q8=0), W.POLICY_LEARNED, tr)
+    assert a["hash"] == b["hash"]
+
+
+def test_ablate_predicted_length_ignores_the_prediction(orc):
+    wl = W.replica_sweep()
+    tr = orc.gen_trace(wl.trace, 2000, replica=3)
+    noisy = dict(tr)
+    rng = np.random.default_rng(0)
+    noisy["pred_out"] = np.clip(tr["pred_out"] * rng.integers(1, 9, tr["pred_out"].size), 1, 1 << 17).astype(np.int32)
+    cc = W.CALIBRATED.replace(ablate=W.ABLATE_PREDICTED_LENGTH)
+    a = orc.simulate(wl.sim, cc, W.POLICY_LEARNED, tr)
+    b = orc.simulate(wl.sim, cc, W.POLICY_LEARNED, noisy)
+    assert a["hash"] == b["hash"]
+    c = orc.simulate(wl.sim, W.CALIBRATED, W.POLICY_LEARNED, noisy)
+    d = orc.simulate(wl.sim, W.CALIBRATED, W.POLICY_LEARNED, tr)
+    assert c["hash"] != d["hash"]
+
+
+def test_ablation_mask_bounds(orc):
+    wl = W.single_replica()
+    tr = orc.gen_trace(wl.trace, 10)
+    assert orc.simulate(wl.sim, W.CALIBRATED.replace(ablate=8), 0, tr)["status"] == orc.EINVAL
+    assert orc.simulate(wl.sim, W.CALIBRATED, 5, tr)["status"] == orc.EINVAL
