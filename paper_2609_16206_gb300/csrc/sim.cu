@@ -77,6 +77,29 @@ __device__ __forceinline__ uint64_t div_recip(uint64_t num, uint64_t d, uint64_t
     return q;
 }
 
+// floor(x / d) for 0 <= x < 2^56 and 0 < d < 2^37: an fp32 estimate from
+// 32-bit conversions, then exact integer correction (the estimate is within a
+// few units of the quotient whenever the quotient is below 2^20, the only
+// case the simulator asks for; larger quotients fall back to division).
+__device__ __forceinline__ int64_t floor_div_small(int64_t x, int64_t d)
+{
+    const float xf = fmaf(__uint2float_rn((uint32_t)(x >> 24)), 16777216.0f, __uint2float_rn((uint32_t)(x & 0xFFFFFF)));
+    const float df = fmaf(__uint2float_rn((uint32_t)(d >> 24)), 16777216.0f, __uint2float_rn((uint32_t)(d & 0xFFFFFF)));
+    const float qf = __fdividef(xf, df);
+    if (!(qf < 1048576.0f)) return x / d;
+    int64_t q = (int64_t)__float2int_rz(qf);
+    int64_t r = x - q * d;
+    while (r < 0) {
+        --q;
+        r += d;
+    }
+    while (r >= d) {
+        ++q;
+        r -= d;
+    }
+    return q;
+}
+
 // floor(x / kv_div) for 0 <= x < 2^32 with magic = ceil(2^64 / kv_div), exact
 __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
 {
@@ -137,7 +160,7 @@ __device__ __forceinline__ int warp_argmin(uint64_t v)
 }
 
 struct Decode {
-    int64_t step_end, step_idx, kv_res, kv_rsv, R, ohat, steps;
+    int64_t step_end, step_idx, kv_res, kv_rsv, R, ohat;
     uint64_t pend_top, act_top;
     int32_t n_act, q, pend_n, act_n, w_head, w_n;
     bool stepping;
@@ -155,13 +178,27 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
         // the general handler below then runs once for all of them together.
         const int64_t tp = s.pend_n > 0 ? (int64_t)(s.pend_top >> kKeyBits) : kNever;
         const int64_t limit = tp <= T ? tp - 1 : T;  // plain step ends lie at or before limit
-        while (s.stepping && s.step_end <= limit && s.w_n == 0 &&
-               (int64_t)(s.act_top >> kKeyBits) != s.step_idx + 1) {
-            s.step_idx += 1;
-            s.kv_res += s.n_act;
-            s.R -= s.n_act;
-            if (++s.steps > P.max_steps) return CTR_ETIMEOUT;
-            s.step_end += P.dec_base + P.dec_seq * s.n_act + kv_term(s.kv_res, P);
+        // The run is taken in closed form: while the floor(KV / kv_div) term of
+        // the step time is unchanged every step lasts S, so the number of plain
+        // ends is the least of the steps before the next completion, the steps
+        // before that term changes, and the steps that end by the limit.
+        while (s.stepping && s.step_end <= limit && s.w_n == 0) {
+            const int64_t m_fin = (int64_t)(s.act_top >> kKeyBits) - s.step_idx - 1;  // <= 2^20
+            if (m_fin <= 0) break;
+            const int64_t n = s.n_act;
+            const int64_t q1 = kv_term(s.kv_res + n, P);  // KV term of the next step
+            const int64_t S = P.dec_base + P.dec_seq * n + q1;
+            const int64_t room = (q1 + 1) * P.kv_div - 1 - s.kv_res;  // the term stays q1 while j n <= room
+            const int64_t m_kv = n <= kRecipN ? (int64_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n]))
+                                              : room / n;
+            int64_t m = m_fin < m_kv ? m_fin : m_kv;
+            const int64_t span = limit - s.step_end;  // plain end j happens at step_end + (j - 1) S <= limit
+            if ((m - 1) * S > span) m = floor_div_small(span, S) + 1;
+            s.step_idx += m;
+            s.kv_res += m * n;
+            s.R -= m * n;
+            if (s.step_idx + 1 > P.max_steps) return CTR_ETIMEOUT;
+            s.step_end += m * S;
             if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
         }
         const int64_t te = s.stepping ? s.step_end : kNever;
@@ -216,7 +253,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 admitted += 1;
             }
             if (s.n_act > 0) {
-                if (++s.steps > P.max_steps) return CTR_ETIMEOUT;
+                if (s.step_idx + 1 > P.max_steps) return CTR_ETIMEOUT;  // steps started on this instance
                 s.step_end = tev + P.dec_base + P.dec_seq * s.n_act + kv_term(s.kv_res, P);
                 if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
                 s.stepping = true;
@@ -334,7 +371,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
         bool live = has_row && valid;
 
         Decode s;
-        s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.R = 0; s.ohat = 0; s.steps = 0;
+        s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.R = 0; s.ohat = 0;
         s.pend_top = kEmpty; s.act_top = kEmpty;
         s.n_act = 0; s.q = 0; s.pend_n = 0; s.act_n = 0; s.w_head = 0; s.w_n = 0;
         s.stepping = false;
