@@ -383,7 +383,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "7c3503c6a7cd87ee": {"warp_inst": 275808953445, "dram_bytes": 33.38e9 + 23.55e9},
+    "9d5bb78182552c4d": {"warp_inst": 202745358987, "dram_bytes": 35.34e9 + 24.70e9},
 }
 
 
