@@ -70,7 +70,8 @@ class _SimCfg(C.Structure):
 class _Consts(C.Structure):
     _fields_ = [("tau_pre0", C.c_int64), ("tau_pre", C.c_int64), ("tau_dec", C.c_int64), ("w_q", C.c_int64),
                 ("w_b_q8", C.c_int64), ("w_s_q8", C.c_int64), ("rho_q8", C.c_int64),
-                ("sigma_q8", C.c_int64 * 4), ("ablate", C.c_int64)]
+                ("sigma_q8", C.c_int64 * 4), ("ablate", C.c_int64),
+                ("proxy_backlog", C.c_int64), ("poll_us", C.c_int64)]
 
 
 class Stats(C.Structure):
@@ -171,6 +172,8 @@ def _consts(cc) -> _Consts:
     for i in range(4):
         s.sigma_q8[i] = int(sig[i])
     s.ablate = int(getattr(cc, "ablate", 0))
+    s.proxy_backlog = int(getattr(cc, "proxy_backlog", 0))
+    s.poll_us = int(getattr(cc, "poll_us", 0))
     return s
 
 

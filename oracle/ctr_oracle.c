@@ -326,6 +326,8 @@ typedef struct {
     int64_t tau_pre0, tau_pre, tau_dec, w_q;
     int64_t w_b_q8, w_s_q8, rho_q8, sigma_q8[4];
     int64_t ablate; /* bit 0: predicted length, bit 1: KV pressure, bit 2: SLO class (sec. V-F) */
+    int64_t proxy_backlog; /* 1: backlog from the proxy's priced in-flight ledger (sec. IV-A, VI) */
+    int64_t poll_us;       /* > 0: KV occupancy seen as polled every poll_us (sec. IV-A); 0: live */
 } orc_consts;
 
 typedef struct {
@@ -425,8 +427,10 @@ typedef struct {
     int64_t** committed; int64_t* n_committed;
     int64_t** fifo; int64_t* fifo_head; int64_t* fifo_tail;
     int64_t* stepping; int64_t* steps;
-    /* per prefill instance */
-    int64_t* busy; int64_t* inflight;
+    /* per prefill instance: in-flight (routed, prefill not ended) request lists */
+    int64_t* busy; int64_t* inflight; int64_t** pre_list;
+    /* KV occupancy of each decode instance at the last poll instant */
+    int64_t* polled_kv;
     heap_t heap;
     orc_stats* st;
     int64_t* admitted;
@@ -593,6 +597,33 @@ static void p2_candidates(int64_t k, int64_t t, int64_t np, int64_t c[2])
     p2_pair(w[2], w[3], np, c);
 }
 
+/* Backlog as the deployed proxy sees it [reading: sec. IV-A's in-flight
+ * ledger "yielding seconds-of-backlog", priced with the router's own
+ * constants as sec. VI describes]: the sum over requests routed to the
+ * instance and still in flight there of their priced work, each priced once
+ * at admission and never decremented.  Prefill: tau_pre0 + tau_pre * p until
+ * the prefill ends; decode: o_hat * tau_dec until the request completes (o_hat
+ * taken as 0 when the predicted length is ablated).  Saturates at 2^40. */
+static int64_t proxy_backlog_pre(const sim_t* s, int64_t i)
+{
+    int64_t b = 0;
+    for (int64_t m = 0; m < s->inflight[i]; ++m) {
+        b += s->cc->tau_pre0 + (int64_t)s->p[s->pre_list[i][m]] * s->cc->tau_pre;
+        if (b >= B_CLAMP) return B_CLAMP;
+    }
+    return b;
+}
+static int64_t proxy_backlog_dec(const sim_t* s, int64_t d)
+{
+    if (s->cc->ablate & 1) return 0;
+    int64_t b = 0;
+    for (int64_t m = 0; m < s->n_committed[d]; ++m) {
+        b += (int64_t)s->oh[s->committed[d][m]] * s->cc->tau_dec;
+        if (b >= B_CLAMP) return B_CLAMP;
+    }
+    return b;
+}
+
 /* Route request k at time t (Algorithm 1) and commit it. */
 static int route(sim_t* s, int64_t k, int64_t t)
 {
@@ -617,6 +648,7 @@ static int route(sim_t* s, int64_t k, int64_t t)
                 int64_t b = s->busy[i] - t;
                 if (b < 0) b = 0;
                 if (b > B_CLAMP) b = B_CLAMP;
+                if (cc->proxy_backlog) b = proxy_backlog_pre(s, i);
                 int64_t own = cc->tau_pre0 + pk * cc->tau_pre;
                 int64_t load = cc->w_b_q8 * b + cc->w_s_q8 * own;
                 cost_p[i] = load * sig + cc->w_q * q * 65536;
@@ -630,7 +662,10 @@ static int route(sim_t* s, int64_t k, int64_t t)
                 int64_t na = dec_active(s, d);
                 int64_t res = dec_resident(s, d);
                 int64_t b = decode_backlog(dec_remaining(s, d), step_time(cfg, na, res), na);
-                int64_t press = ((res + pk + oh_f) * 65536) / cfg->kv_cap;
+                if (cc->proxy_backlog) b = proxy_backlog_dec(s, d);
+                /* press+ from the occupancy the router sees: live, or the last poll */
+                int64_t seen = cc->poll_us > 0 ? s->polled_kv[d] : res;
+                int64_t press = ((seen + pk + oh_f) * 65536) / cfg->kv_cap;
                 if (press > P_CLAMP) press = P_CLAMP;
                 if (cc->ablate & 2) press = 0;
                 int64_t own = oh_f * cc->tau_dec;
@@ -661,7 +696,7 @@ static int route(sim_t* s, int64_t k, int64_t t)
     int64_t ready = end + cfg->xfer_per_tok * pk;
     if (ready >= T_LIMIT) return ORC_EOVERFLOW;
     s->busy[ip] = end;
-    s->inflight[ip] += 1;
+    s->pre_list[ip][s->inflight[ip]++] = k;
     if (s->inflight[ip] > s->st->max_prefill) s->st->max_prefill = s->inflight[ip];
     if (cfg->cap_prefill > 0 && s->inflight[ip] > cfg->cap_prefill) return ORC_EOVERFLOW;
     ev_t e1 = {end, EV_PREFILL_END, k, ip};
@@ -706,6 +741,8 @@ static int validate_cfg(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t po
     if (cfg->n_classes < 1 || cfg->n_classes > 4) return ORC_EINVAL;
     if (policy < 0 || policy > 4) return ORC_EINVAL;
     if (cc->ablate < 0 || cc->ablate > 7) return ORC_EINVAL;
+    if (cc->proxy_backlog < 0 || cc->proxy_backlog > 1) return ORC_EINVAL;
+    if (cc->poll_us < 0 || cc->poll_us > ARR_LIMIT) return ORC_EINVAL;
     if (cc->w_b_q8 < 0 || cc->w_b_q8 > 1023 || cc->w_s_q8 < 0 || cc->w_s_q8 > 1023) return ORC_EINVAL;
     if (cc->rho_q8 < 0 || cc->rho_q8 > 1023) return ORC_EINVAL;
     for (int i = 0; i < 4; ++i)
@@ -749,10 +786,17 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
     s.steps = (int64_t*)calloc((size_t)nd, 8);
     s.busy = (int64_t*)calloc((size_t)np, 8);
     s.inflight = (int64_t*)calloc((size_t)np, 8);
+    s.pre_list = (int64_t**)calloc((size_t)np, sizeof(int64_t*));
+    s.polled_kv = (int64_t*)calloc((size_t)nd, 8);
     rc = ORC_OK;
     if (!s.stage || !s.gen || !s.dec_of || !s.admitted || !s.committed || !s.fifo || !s.n_committed ||
-        !s.fifo_head || !s.fifo_tail || !s.stepping || !s.steps || !s.busy || !s.inflight)
+        !s.fifo_head || !s.fifo_tail || !s.stepping || !s.steps || !s.busy || !s.inflight || !s.pre_list ||
+        !s.polled_kv)
         rc = ORC_ENOMEM;
+    for (int64_t i = 0; i < np && rc == ORC_OK; ++i) {
+        s.pre_list[i] = (int64_t*)calloc((size_t)nn, 8);
+        if (!s.pre_list[i]) rc = ORC_ENOMEM;
+    }
     for (int64_t d = 0; d < nd && rc == ORC_OK; ++d) {
         s.committed[d] = (int64_t*)calloc((size_t)nn, 8);
         s.fifo[d] = (int64_t*)calloc((size_t)nn, 8);
@@ -761,10 +805,12 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
     for (int64_t k = 0; k < n; ++k) t_first[k] = t_done[k] = pre_end[k] = t_ready[k] = -1;
 
     int64_t ia = 0;
+    int64_t next_poll = 0; /* occupancy polls at 0, poll_us, 2 poll_us, ... while arrivals remain */
     while (rc == ORC_OK) {
         int64_t t = INT64_MAX;
         if (s.heap.n > 0) t = s.heap.a[0].t;
         if (ia < n && arr[ia] < t) t = arr[ia];
+        if (ia < n && cc->poll_us > 0 && next_poll < t) t = next_poll;
         if (t == INT64_MAX) break;
         /* (1) step ends, prefill ends and KV-ready events at t, KV-ready in
          * order of request index [reading: equal-time order] */
@@ -774,7 +820,9 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
             if (e.kind == EV_STEP_END) {
                 on_step_end(&s, e.inst, t);
             } else if (e.kind == EV_PREFILL_END) {
-                s.inflight[e.inst] -= 1;
+                int64_t i = 0;
+                while (s.pre_list[e.inst][i] != e.k) ++i;
+                s.pre_list[e.inst][i] = s.pre_list[e.inst][--s.inflight[e.inst]];
             } else {
                 int64_t d = e.inst;
                 s.stage[e.k] = ST_WAITING;
@@ -789,6 +837,12 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
         for (int64_t d = 0; d < nd && rc == ORC_OK; ++d)
             if (!s.stepping[d]) rc = admit_and_start(&s, d, t);
         if (rc) break;
+        /* the occupancy poll at t sees the state after every event at t and
+         * before the arrivals at t [reading: equal-time order] */
+        if (cc->poll_us > 0 && t == next_poll) {
+            for (int64_t d = 0; d < nd; ++d) s.polled_kv[d] = dec_resident(&s, d);
+            next_poll += cc->poll_us;
+        }
         /* (3) arrivals at t, in order of request index */
         while (ia < n && arr[ia] == t && rc == ORC_OK) {
             rc = route(&s, ia, t);
@@ -803,7 +857,9 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
     }
     free(s.stage); free(s.gen); free(s.dec_of); free(s.admitted); free(s.committed); free(s.fifo);
     free(s.n_committed); free(s.fifo_head); free(s.fifo_tail); free(s.stepping); free(s.steps);
-    free(s.busy); free(s.inflight); free(s.heap.a);
+    for (int64_t i = 0; i < np; ++i)
+        if (s.pre_list) free(s.pre_list[i]);
+    free(s.busy); free(s.inflight); free(s.pre_list); free(s.polled_kv); free(s.heap.a);
     return rc;
 }
 

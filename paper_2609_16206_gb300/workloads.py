@@ -28,6 +28,7 @@ POLICY_LEARNED, POLICY_RR, POLICY_JSQ, POLICY_HEURISTIC, POLICY_LEARNED_P2 = 0, 
 POLICY_NAMES = {POLICY_LEARNED: "learned", POLICY_RR: "round_robin", POLICY_JSQ: "least_loaded",
                 POLICY_HEURISTIC: "length_heuristic", POLICY_LEARNED_P2: "learned_power_of_two"}
 ABLATE_PREDICTED_LENGTH, ABLATE_PRESSURE, ABLATE_SLO = 1, 2, 4
+PROXY_POLL_US = 50_000               # the deployed proxy's occupancy poll period (sec. IV-A)
 ALL_POLICIES = (POLICY_LEARNED, POLICY_RR, POLICY_JSQ, POLICY_HEURISTIC)
 
 
@@ -103,6 +104,8 @@ class CostConsts:
     rho_q8: int = 256
     sigma_q8: tuple = (512, 256, 256, 256)
     ablate: int = 0                  # ABLATE_* bits: features replaced by their neutral value
+    proxy_backlog: int = 0           # 1: backlog from the proxy's priced in-flight ledger, 0: true remaining work
+    poll_us: int = 0                 # > 0: KV occupancy polled every poll_us (the proxy's 50 ms); 0: live
 
     def replace(self, **kw) -> "CostConsts":
         return dataclasses.replace(self, **kw)
@@ -145,6 +148,11 @@ def large_pool(n_replicas: int = 16384, n_req: int = 50_000, rate_mreq: int = 33
     cc = CostConsts(sigma_q8=(512, 384, 256, 256))
     return SweepWorkload(f"large_pool_4p28d_{n_replicas}x{n_req}", tc, sc, consts=[cc],
                          n_replicas=n_replicas, n_req=n_req)
+
+
+def as_deployed(cc: CostConsts) -> CostConsts:
+    """The same constants with the deployed proxy's signals: ledger backlog and a 50 ms occupancy poll."""
+    return cc.replace(proxy_backlog=1, poll_us=PROXY_POLL_US)
 
 
 def mispriced_sets(base: CostConsts = CALIBRATED, factors=(0.5, 0.75, 1.5, 2.0)) -> list:
