@@ -371,7 +371,7 @@ def run_ours(args, rank, world, local_rank):
         "e2e": {"value": e2e_value, "unit": "routed requests/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "note": "host trace + scorer inputs copied in, simulate + goodput + score, results copied out"},
-        "gpu_launches": 4 * args.steps,
+        "gpu_launches": 5 * args.steps,  # gen, sim, checksum pass, goodput, score
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)
@@ -383,7 +383,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "9d5bb78182552c4d": {"warp_inst": 202745358987, "dram_bytes": 35.34e9 + 24.70e9},
+    "f64f9a4e5f70184c": {"warp_inst": 189399495450, "dram_bytes": 35.78e9 + 25.13e9},
 }
 
 

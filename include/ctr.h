@@ -52,6 +52,10 @@ enum ctr_policy {
 #define CTR_ABLATE_PRESSURE 2u         /* P := 0 */
 #define CTR_ABLATE_SLO 4u              /* sigma := 1.0 (256) for every class */
 
+/* Where the learned router's backlog signal comes from (ctr_cost_consts.backlog_signal). */
+#define CTR_BACKLOG_TRUE 0u  /* the cluster's true remaining work (the simulator's own clock) */
+#define CTR_BACKLOG_PROXY 1u /* the deployed proxy's in-flight ledger priced with the router's constants */
+
 enum ctr_workspace_kind { CTR_WS_SIMULATE = 0 };
 
 /* A batch of requests in structure-of-arrays form: element [r * n_req + k] is
@@ -126,13 +130,25 @@ typedef struct ctr_sim_cfg {
  * with key (0x243F6A88, 0x85A308D3) and counter (k, t lo, t hi, 0x5032) gives
  * u0..u3; a pool of n offers c0 = floor(u n / 2^32) and
  * c1 = (c0 + 1 + floor(u' (n - 1) / 2^32)) mod n (decode (u0, u1), prefill
- * (u2, u3)), and the cheaper one wins (ties to the lower index). */
+ * (u2, u3)), and the cheaper one wins (ties to the lower index).
+ * Signals as the deployed proxy sees them (sec. IV-A; sec. VI explains why
+ * they matter for calibration):
+ *   backlog_signal = CTR_BACKLOG_PROXY replaces B_p and B_d by the in-flight
+ *     ledger, each request priced once when routed and dropped when it leaves:
+ *     B_p = min(2^40, sum over requests whose prefill on p has not ended of
+ *     tau_pre0 + tau_pre * p), B_d = min(2^40, tau_dec * sum of o_hat over
+ *     requests routed to d and not completed) (0 when o_hat is ablated).
+ *   occupancy_poll_us = D > 0 makes P use the resident KV of d as it was at
+ *     the last poll instant floor(t / D) * D (after every event at that
+ *     instant) instead of its live value; 0 = live. */
 typedef struct ctr_cost_consts {
     int64_t tau_pre0_us, tau_pre_us, tau_dec_us; /* 0..2^20 */
     int64_t w_q_us;                              /* 0..2^20, us per in-flight request */
     int32_t w_b_q8, w_s_q8, rho_q8;              /* 0..1023 */
     int32_t sigma_q8[4];                         /* 0..1023 */
     uint32_t ablate;                             /* CTR_ABLATE_* bits, 0 = every feature */
+    uint32_t backlog_signal;                     /* CTR_BACKLOG_TRUE or CTR_BACKLOG_PROXY */
+    int64_t occupancy_poll_us;                   /* 0..2^39; 0 = live occupancy */
 } ctr_cost_consts;
 
 /* ctr_gen_trace -- synthetic request trace (Table 1 length profiles as

@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 2;
+constexpr int kAbiVersion = 3;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -54,6 +54,8 @@ bool valid_consts(const ctr_cost_consts& k)
     for (int i = 0; i < 4; ++i)
         if (!in_range(k.sigma_q8[i], 0, 1023)) return false;
     if (k.ablate > 7u) return false;
+    if (k.backlog_signal > CTR_BACKLOG_PROXY) return false;
+    if (!in_range(k.occupancy_poll_us, 0, kArrivalLimit)) return false;
     return true;
 }
 
@@ -251,6 +253,9 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
         d.rho = k.rho_q8;
         for (int c = 0; c < 4; ++c) d.sigma[c] = k.sigma_q8[c];
         d.ablate = k.ablate;
+        d.proxy = k.backlog_signal;
+        d.poll_us = k.occupancy_poll_us;
+        d.poll_recip = k.occupancy_poll_us > 0 ? ~0ull / (uint64_t)k.occupancy_poll_us : 0;
     }
 
     p.slot_bytes = sim_slot_bytes(*cfg, &p.off_act, &p.off_wait, &p.cap_pr);

@@ -62,6 +62,9 @@ struct ConstsDev {
     int64_t tau_pre0, tau_pre, tau_dec, w_q;
     int32_t w_b, w_s, rho, sigma[4];
     uint32_t ablate;
+    uint32_t proxy;       // backlog from the priced in-flight ledger
+    int64_t poll_us;      // > 0: occupancy polled on this period
+    uint64_t poll_recip;  // floor((2^64 - 1) / poll_us)
 };
 
 struct SimParams {

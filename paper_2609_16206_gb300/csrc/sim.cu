@@ -22,7 +22,8 @@
 // Per-lane structures live in the workspace slot of the warp, interleaved
 // [entry][lane] so that the lanes' heap tops share cache lines: a min-heap of
 // pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
-// lanes use the same region as their in-flight ring of prefill end times),
+// lanes use the same region as their in-flight ring of prefill end times,
+// packed with the prompt length as end << 21 | p),
 // a min-heap of active requests keyed by finishing step (finish << 23 | k),
 // and a FIFO ring of KV-ready requests awaiting admission.  Heap tops are
 // cached in registers, so a plain decode step touches no memory.
@@ -38,6 +39,8 @@ constexpr int64_t kNever = INT64_MAX;
 constexpr int64_t kBacklogClamp = int64_t(1) << 40;
 constexpr int64_t kPressureClamp = int64_t(1) << 18;
 constexpr int kRecipN = 1024;  // batch sizes with a tabulated reciprocal
+constexpr int kRingPBits = 21;  // prefill ring entry: end << 21 | p (p <= 2^20)
+constexpr int64_t kRingPMask = (int64_t(1) << kRingPBits) - 1;
 
 // floor((2^64 - 1) / n) for n = 1..kRecipN, for the decode backlog's division
 // by the batch size (built at compile time, read through the read-only path)
@@ -168,7 +171,7 @@ struct Decode {
 
 // Advance one decode instance through every event at times <= T.
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
-                                              uint32_t* wait, int64_t tb, int64_t ob, uint64_t& h)
+                                              uint32_t* wait, int64_t tb, int64_t ob)
 {
     for (;;) {
         // Plain step ends first, in a tight loop: the step ends by T, no request
@@ -221,7 +224,6 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 s.kv_rsv -= pk + ok;
                 s.ohat -= ohk;
                 P.t_done[ob + k] = tev;
-                h += hterm(k, 3, (uint64_t)tev);
             }
         }
         // (2) KV-ready requests join the waiting FIFO in (time, index) order
@@ -261,7 +263,6 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 for (int i = 0; i < admitted; ++i) {  // first token at the end of this step
                     const uint32_t k = wait[pos * kWarp];
                     P.t_first[ob + k] = s.step_end;
-                    h += hterm(k, 2, (uint64_t)s.step_end);
                     pos = pos + 1 == P.cap_wait ? 0 : pos + 1;
                 }
             }
@@ -324,8 +325,10 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // workload have the same number of requests, so the groups walk their
 // arrivals in lockstep (request k of every row at once, each at its own time);
 // the per-lane event loops, the per-group argmins and the commits are
-// independent across groups.
-template <int G>
+// independent across groups.  kSignals compiles in the deployed proxy's
+// signals (ledger backlog, polled occupancy); the host launches that
+// instantiation only when some constant set asks for one of them.
+template <int G, bool kSignals>
 __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __grid_constant__ SimParams P)
 {
     constexpr int kRowsPerWarp = 32 / G;
@@ -375,8 +378,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
         s.pend_top = kEmpty; s.act_top = kEmpty;
         s.n_act = 0; s.q = 0; s.pend_n = 0; s.act_n = 0; s.w_head = 0; s.w_n = 0;
         s.stepping = false;
-        int64_t busy = 0, ring_front = kNever;  // prefill lanes
+        int64_t busy = 0, ring_front = kNever;  // prefill lanes: ring_front = front entry (end << 21 | p)
+        int64_t ring_sum_p = 0;                  // prompt tokens of the prefills in the ring
         int32_t ring_head = 0, ring_n = 0;
+        int64_t kv_seen = 0, last_poll = -1;     // decode lanes: occupancy at the last poll instant
         int32_t rr_p = 0, rr_d = 0;
         uint64_t h = 0;
         int err = CTR_OK;
@@ -407,9 +412,22 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                 // 1. advance every instance to the arrival time
                 if (live) {
                     if (is_dec) {
-                        err = decode_advance(s, T, P, pend, act, wait, tb, ob, h);
+                        if (kSignals && cc.poll_us > 0) {
+                            // the router sees the occupancy of the last poll instant floor(T / D) D,
+                            // taken after every event at that instant: advance there first
+                            const int64_t tp = (int64_t)div_recip((uint64_t)T, (uint64_t)cc.poll_us, cc.poll_recip) *
+                                               cc.poll_us;
+                            if (tp > last_poll) {
+                                err = decode_advance(s, tp, P, pend, act, wait, tb, ob);
+                                kv_seen = s.kv_res;
+                                last_poll = tp;
+                            }
+                        }
+                        if (err == CTR_OK) err = decode_advance(s, T, P, pend, act, wait, tb, ob);
                     } else if (is_pre) {
-                        while (ring_n > 0 && ring_front <= T) {
+                        const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
+                        while (ring_n > 0 && ring_front <= thr) {
+                            if constexpr (kSignals) ring_sum_p -= ring_front & kRingPMask;
                             ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
                             ring_n -= 1;
                             ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
@@ -428,7 +446,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                     const int64_t sig = (cc.ablate & CTR_ABLATE_SLO) ? 256 : cc.sigma[ck];
                     if (is_pre) {
                         if (learned) {
-                            const int64_t b = busy > T ? busy - T : 0;
+                            int64_t b = busy > T ? busy - T : 0;
+                            if (kSignals && cc.proxy) {  // the ledger: tau_pre0 + tau_pre p per prefill not yet ended
+                                b = cc.tau_pre0 * (int64_t)ring_n + cc.tau_pre * ring_sum_p;
+                                if (b > kBacklogClamp) b = kBacklogClamp;
+                            }
                             const int64_t load = cc.w_b * b + cc.w_s * (cc.tau_pre0 + pk * cc.tau_pre);
                             cost = (uint64_t)(load * sig + cc.w_q * (int64_t)ring_n * 65536);
                         } else {
@@ -449,7 +471,12 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                                                                       : lo / nd);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            int64_t press = (int64_t)div_recip((uint64_t)(s.kv_res + pk + oh_f) << 16,
+                            if (kSignals && cc.proxy) {  // the ledger: tau_dec o_hat per request routed here and not done
+                                b = (cc.ablate & CTR_ABLATE_PREDICTED_LENGTH) ? 0 : cc.tau_dec * s.ohat;
+                                if (b > kBacklogClamp) b = kBacklogClamp;
+                            }
+                            const int64_t kv = kSignals && cc.poll_us > 0 ? kv_seen : s.kv_res;
+                            int64_t press = (int64_t)div_recip((uint64_t)(kv + pk + oh_f) << 16,
                                                                (uint64_t)P.kv_cap, P.kv_cap_recip);
                             if (press > kPressureClamp) press = kPressureClamp;
                             if (cc.ablate & CTR_ABLATE_PRESSURE) press = 0;
@@ -506,9 +533,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                         busy = end;
                         int pos = ring_head + ring_n;
                         if (pos >= P.cap_ring) pos -= P.cap_ring;
-                        ring[pos * kWarp] = end;
-                        if (ring_n == 0) ring_front = end;
+                        const int64_t e = (end << kRingPBits) | pk;
+                        ring[pos * kWarp] = e;
+                        if (ring_n == 0) ring_front = e;
                         ring_n += 1;
+                        if constexpr (kSignals) ring_sum_p += pk;
                     }
                 }
                 ready = __shfl_sync(kFull, ready, ip, G);
@@ -522,17 +551,19 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                         s.ohat += ohk;
                     }
                 }
-                if (live && gl == 0) h += hterm(k, 1, ((uint64_t)ip << 8) | (uint64_t)id);
                 if (gl == j) my_route = ((uint32_t)ip << 8) | (uint32_t)id;
                 if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
             }
             if (mine && live) {
+                // the routing term of the row checksum, all lanes at once (the
+                // first-token and completion terms are added by hash_kernel)
+                h += hterm(kl, 1, (uint64_t)my_route);
                 if (P.i_pre) P.i_pre[ob + kl] = (uint8_t)(my_route >> 8);
                 if (P.i_dec) P.i_dec[ob + kl] = (uint8_t)(my_route & 0xFF);
             }
         }
         // drain: every remaining event
-        if (live && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob, h);
+        if (live && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob);
 
 #pragma unroll
         for (int off = G / 2; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off, G);
@@ -544,6 +575,36 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
             P.row_status[row] = status;
             P.row_hash[row] = status == CTR_OK ? h : 0;
         }
+    }
+}
+
+// The first-token and completion terms of the row checksum, one block per
+// row over the simulator's outputs (coalesced; cheaper than hashing inside
+// the diverged event handlers).  Rows that failed keep the checksum 0.
+constexpr int kHashThreads = 256;
+__global__ void __launch_bounds__(kHashThreads) hash_kernel(const __grid_constant__ SimParams P)
+{
+    __shared__ uint64_t part[kHashThreads / 32];
+    for (int64_t row = blockIdx.x; row < P.n_rows; row += gridDim.x) {
+        if (P.row_status[row] != CTR_OK) continue;  // block-uniform
+        const int64_t ob = row * P.n_req;
+        uint64_t h = 0;
+#pragma unroll 4
+        for (int64_t k = threadIdx.x; k < P.n_req; k += kHashThreads) {
+            const int64_t tf = __ldcs(&P.t_first[ob + k]);
+            const int64_t td = __ldcs(&P.t_done[ob + k]);
+            h += hterm(k, 2, (uint64_t)tf) + hterm(k, 3, (uint64_t)td);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off);
+        if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = h;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            uint64_t t = 0;
+            for (int w = 0; w < kHashThreads / 32; ++w) t += part[w];
+            P.row_hash[row] += t;
+        }
+        __syncthreads();  // part[] is reused by the next row
     }
 }
 
@@ -573,8 +634,10 @@ int sim_max_resident_warps(int* warps_per_block, int* blocks)
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
     // the smallest occupancy over the group widths, so one workspace size fits every launch
     per_sm = 1 << 30;
-    const void* kernels[4] = {(const void*)sim_kernel<4>, (const void*)sim_kernel<8>, (const void*)sim_kernel<16>,
-                              (const void*)sim_kernel<32>};
+    const void* kernels[8] = {(const void*)sim_kernel<4, false>, (const void*)sim_kernel<8, false>,
+                              (const void*)sim_kernel<16, false>, (const void*)sim_kernel<32, false>,
+                              (const void*)sim_kernel<4, true>, (const void*)sim_kernel<8, true>,
+                              (const void*)sim_kernel<16, true>, (const void*)sim_kernel<32, true>};
     for (const void* k : kernels) {
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_g, k, kWarpsPerBlock * 32, 0) != cudaSuccess)
             return 0;
@@ -588,11 +651,22 @@ int sim_max_resident_warps(int* warps_per_block, int* blocks)
 cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
 {
     (void)warps_per_block;
-    switch (sim_group_width(p.n_pre + p.n_dec)) {
-    case 4: sim_kernel<4><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
-    case 8: sim_kernel<8><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
-    case 16: sim_kernel<16><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
-    default: sim_kernel<32><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p); break;
+    bool signals = false;
+    for (int i = 0; i < p.n_sets; ++i) signals = signals || p.sets[i].proxy != 0 || p.sets[i].poll_us > 0;
+    const dim3 grid(blocks), block(kWarpsPerBlock * 32);
+    switch (sim_group_width(p.n_pre + p.n_dec) * 2 + (signals ? 1 : 0)) {
+    case 8: sim_kernel<4, false><<<grid, block, 0, stream>>>(p); break;
+    case 9: sim_kernel<4, true><<<grid, block, 0, stream>>>(p); break;
+    case 16: sim_kernel<8, false><<<grid, block, 0, stream>>>(p); break;
+    case 17: sim_kernel<8, true><<<grid, block, 0, stream>>>(p); break;
+    case 32: sim_kernel<16, false><<<grid, block, 0, stream>>>(p); break;
+    case 33: sim_kernel<16, true><<<grid, block, 0, stream>>>(p); break;
+    case 64: sim_kernel<32, false><<<grid, block, 0, stream>>>(p); break;
+    default: sim_kernel<32, true><<<grid, block, 0, stream>>>(p); break;
+    }
+    if (p.n_rows > 0) {
+        const int64_t hb = p.n_rows < (int64_t)blocks * 8 ? p.n_rows : (int64_t)blocks * 8;
+        hash_kernel<<<(unsigned)hb, kHashThreads, 0, stream>>>(p);
     }
     return cudaGetLastError();
 }

@@ -66,7 +66,8 @@ class CtrSimCfg(C.Structure):
 class CtrCostConsts(C.Structure):
     _fields_ = [("tau_pre0_us", C.c_int64), ("tau_pre_us", C.c_int64), ("tau_dec_us", C.c_int64),
                 ("w_q_us", C.c_int64), ("w_b_q8", C.c_int32), ("w_s_q8", C.c_int32), ("rho_q8", C.c_int32),
-                ("sigma_q8", C.c_int32 * 4), ("ablate", C.c_uint32)]
+                ("sigma_q8", C.c_int32 * 4), ("ablate", C.c_uint32),
+                ("backlog_signal", C.c_uint32), ("occupancy_poll_us", C.c_int64)]
 
 
 _lock = threading.Lock()
@@ -182,6 +183,8 @@ def consts_array(sets):
         for c in range(4):
             a.sigma_q8[c] = int(sig[c])
         a.ablate = int(getattr(cc, "ablate", 0))
+        a.backlog_signal = int(getattr(cc, "proxy_backlog", 0))
+        a.occupancy_poll_us = int(getattr(cc, "poll_us", 0))
     return arr
 
 

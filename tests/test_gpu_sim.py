@@ -226,3 +226,33 @@ def test_power_of_two_router(orc, wl):
     pols = [W.POLICY_LEARNED_P2, W.POLICY_LEARNED, W.POLICY_RR]
     res = simulate(ctr, wl.sim, [wl.consts[0]], pols, tr, R, N)
     _check_rows(orc, wl.sim, [wl.consts[0]], pols, [host_trace(tr, r) for r in range(R)], res, N)
+
+
+def _signal_sets(base):
+    """True / ledger backlog x live / 50 ms / 7 ms occupancy, plus a mispriced ledger set."""
+    return [base, base.replace(proxy_backlog=1), base.replace(poll_us=W.PROXY_POLL_US), W.as_deployed(base),
+            base.replace(poll_us=7_000, proxy_backlog=1, ablate=W.ABLATE_PREDICTED_LENGTH),
+            W.as_deployed(base).replace(tau_dec_us=base.tau_dec_us // 2, tau_pre0_us=2 * base.tau_pre0_us)]
+
+
+@pytest.mark.parametrize("wl", [W.replica_sweep(), W.large_pool(rate_mreq=34_000), W.single_replica()],
+                         ids=["2p6d", "4p28d", "1p3d"])
+def test_proxy_signals(orc, wl):
+    """Ledger backlog and polled occupancy (sec. IV-A) in one launch with the
+    true signals, every row bit-identical to the oracle."""
+    ctr = need_gpu()
+    R, N = 3, 2500
+    tr = gen(ctr, wl.trace, R, N)
+    sets = _signal_sets(wl.consts[0])
+    pols = [W.POLICY_LEARNED, W.POLICY_LEARNED_P2]
+    res = simulate(ctr, wl.sim, sets, pols, tr, R, N)
+    _check_rows(orc, wl.sim, sets, pols, [host_trace(tr, r) for r in range(R)], res, N)
+
+
+def test_proxy_signals_host_validation():
+    ctr = need_gpu()
+    wl = W.single_replica()
+    tr = gen(ctr, wl.trace, 1, 16)
+    for bad in (dict(proxy_backlog=2), dict(poll_us=-1), dict(poll_us=(1 << 39) + 1)):
+        with pytest.raises(ctr.CtrError):
+            simulate(ctr, wl.sim, [W.CALIBRATED.replace(**bad)], [W.POLICY_LEARNED], tr, 1, 16)
