@@ -64,7 +64,7 @@ class _SimCfg(C.Structure):
                 ("n_classes", C.c_int64), ("ttft", C.c_int64 * 4), ("tpot", C.c_int64 * 4),
                 ("max_steps", C.c_int64),
                 ("cap_pending", C.c_int64), ("cap_waiting", C.c_int64), ("cap_active", C.c_int64),
-                ("cap_prefill", C.c_int64), ("heur_thresh", C.c_int64)]
+                ("cap_prefill", C.c_int64), ("heur_thresh", C.c_int64), ("pre_batch_tokens", C.c_int64)]
 
 
 class _Consts(C.Structure):
@@ -161,6 +161,7 @@ def _sim_cfg(sc) -> _SimCfg:
     s.cap_pending, s.cap_waiting = int(sc.cap_pending), int(sc.cap_waiting)
     s.cap_active, s.cap_prefill = int(sc.cap_active), int(sc.cap_prefill_ring)
     s.heur_thresh = int(sc.heuristic_threshold_tokens)
+    s.pre_batch_tokens = int(getattr(sc, "prefill_batch_tokens", 0))
     return s
 
 

@@ -320,6 +320,7 @@ typedef struct {
     int64_t max_steps;                     /* decode steps allowed per decode instance */
     int64_t cap_pending, cap_waiting, cap_active, cap_prefill; /* 0 = unlimited */
     int64_t heur_thresh;
+    int64_t pre_batch_tokens;              /* 0: serial FCFS prefill; > 0: batched prefill with this token budget */
 } orc_sim_cfg;
 
 typedef struct {
@@ -431,6 +432,10 @@ typedef struct {
     int64_t* busy; int64_t* inflight; int64_t** pre_list;
     /* KV occupancy of each decode instance at the last poll instant */
     int64_t* polled_kv;
+    /* batched prefill: per instance the FIFO of requests not yet in a batch
+     * and the members of the running batch */
+    int64_t** pfifo; int64_t* pfifo_head; int64_t* pfifo_tail;
+    int64_t** prun; int64_t* prun_n; int64_t* prun_end; int64_t* prun_on;
     heap_t heap;
     orc_stats* st;
     int64_t* admitted;
@@ -597,6 +602,68 @@ static void p2_candidates(int64_t k, int64_t t, int64_t np, int64_t c[2])
     p2_pair(w[2], w[3], np, c);
 }
 
+/* Batched prefill (sec. VI: continuous batching "in both stages") [reading]:
+ * an instance runs one batch at a time.  A batch takes, FCFS from the
+ * instance's queue, the head request and then every next request while the
+ * batch's prompt tokens stay within pre_batch_tokens; it lasts
+ * pre_base + pre_per_tok * (sum of its prompts), and each member's KV transfer
+ * starts when the batch ends.  A batch starts when the previous one ends (if
+ * anything waits) or when a request reaches an idle instance. */
+static int start_prefill_batch(sim_t* s, int64_t i, int64_t t)
+{
+    const orc_sim_cfg* cfg = s->cfg;
+    int64_t tokens = 0;
+    s->prun_n[i] = 0;
+    while (s->pfifo_head[i] < s->pfifo_tail[i]) {
+        int64_t j = s->pfifo[i][s->pfifo_head[i]];
+        if (s->prun_n[i] > 0 && tokens + (int64_t)s->p[j] > cfg->pre_batch_tokens) break;
+        tokens += s->p[j];
+        s->prun[i][s->prun_n[i]++] = j;
+        s->pfifo_head[i]++;
+    }
+    int64_t end = t + cfg->pre_base + cfg->pre_per_tok * tokens;
+    if (end >= T_LIMIT) return ORC_EOVERFLOW;
+    ev_t e = {end, EV_PREFILL_END, -1, i};
+    if (heap_push(&s->heap, e)) return ORC_ENOMEM;
+    for (int64_t m = 0; m < s->prun_n[i]; ++m) {
+        int64_t j = s->prun[i][m];
+        int64_t ready = end + cfg->xfer_per_tok * (int64_t)s->p[j];
+        if (ready >= T_LIMIT) return ORC_EOVERFLOW;
+        ev_t r = {ready, EV_KV_READY, j, s->dec_of[j]};
+        if (heap_push(&s->heap, r)) return ORC_ENOMEM;
+        s->pre_end[j] = end;
+        s->t_ready[j] = ready;
+    }
+    s->prun_on[i] = 1;
+    s->prun_end[i] = end;
+    return ORC_OK;
+}
+
+/* True prefill backlog under batching [reading]: the time until the instance
+ * would have served everything committed to it if nothing else arrived --
+ * the rest of the running batch, then the queue cut into batches by the same
+ * FCFS token-budget rule, each costing base + per_tok * its prompt tokens.
+ * Saturates at 2^40. */
+static int64_t batched_backlog_pre(const sim_t* s, int64_t i, int64_t t)
+{
+    const orc_sim_cfg* cfg = s->cfg;
+    int64_t b = s->prun_on[i] && s->prun_end[i] > t ? s->prun_end[i] - t : 0;
+    int64_t m = s->pfifo_head[i];
+    while (m < s->pfifo_tail[i]) {
+        int64_t tokens = 0, members = 0;
+        while (m < s->pfifo_tail[i]) {
+            int64_t pj = s->p[s->pfifo[i][m]];
+            if (members > 0 && tokens + pj > cfg->pre_batch_tokens) break;
+            tokens += pj;
+            members++;
+            m++;
+        }
+        b += cfg->pre_base + cfg->pre_per_tok * tokens;
+        if (b >= B_CLAMP) return B_CLAMP;
+    }
+    return b;
+}
+
 /* Backlog as the deployed proxy sees it [reading: sec. IV-A's in-flight
  * ledger "yielding seconds-of-backlog", priced with the router's own
  * constants as sec. VI describes]: the sum over requests routed to the
@@ -648,6 +715,7 @@ static int route(sim_t* s, int64_t k, int64_t t)
                 int64_t b = s->busy[i] - t;
                 if (b < 0) b = 0;
                 if (b > B_CLAMP) b = B_CLAMP;
+                if (cfg->pre_batch_tokens > 0) b = batched_backlog_pre(s, i, t);
                 if (cc->proxy_backlog) b = proxy_backlog_pre(s, i);
                 int64_t own = cc->tau_pre0 + pk * cc->tau_pre;
                 int64_t load = cc->w_b_q8 * b + cc->w_s_q8 * own;
@@ -691,20 +759,31 @@ static int route(sim_t* s, int64_t k, int64_t t)
         }
     }
 
-    int64_t start = s->busy[ip] > t ? s->busy[ip] : t;
-    int64_t end = start + cfg->pre_base + cfg->pre_per_tok * pk;
-    int64_t ready = end + cfg->xfer_per_tok * pk;
-    if (ready >= T_LIMIT) return ORC_EOVERFLOW;
-    s->busy[ip] = end;
+    s->stage[k] = ST_PENDING;
+    s->dec_of[k] = id;
     s->pre_list[ip][s->inflight[ip]++] = k;
     if (s->inflight[ip] > s->st->max_prefill) s->st->max_prefill = s->inflight[ip];
     if (cfg->cap_prefill > 0 && s->inflight[ip] > cfg->cap_prefill) return ORC_EOVERFLOW;
-    ev_t e1 = {end, EV_PREFILL_END, k, ip};
-    ev_t e2 = {ready, EV_KV_READY, k, id};
-    if (heap_push(&s->heap, e1) || heap_push(&s->heap, e2)) return ORC_ENOMEM;
-
-    s->stage[k] = ST_PENDING;
-    s->dec_of[k] = id;
+    if (cfg->pre_batch_tokens > 0) {
+        /* batched: join the instance's queue; an idle instance starts a batch at once */
+        s->pfifo[ip][s->pfifo_tail[ip]++] = k;
+        if (!s->prun_on[ip]) {
+            int rc = start_prefill_batch(s, ip, t);
+            if (rc) return rc;
+        }
+    } else {
+        /* serial FCFS: the prefill's start, end and KV-ready time in closed form */
+        int64_t start = s->busy[ip] > t ? s->busy[ip] : t;
+        int64_t end = start + cfg->pre_base + cfg->pre_per_tok * pk;
+        int64_t ready = end + cfg->xfer_per_tok * pk;
+        if (ready >= T_LIMIT) return ORC_EOVERFLOW;
+        s->busy[ip] = end;
+        ev_t e1 = {end, EV_PREFILL_END, k, ip};
+        ev_t e2 = {ready, EV_KV_READY, k, id};
+        if (heap_push(&s->heap, e1) || heap_push(&s->heap, e2)) return ORC_ENOMEM;
+        s->pre_end[k] = end;
+        s->t_ready[k] = ready;
+    }
     s->committed[id][s->n_committed[id]++] = k;
     int64_t pend = dec_pending(s, id);
     if (pend > s->st->max_pending) s->st->max_pending = pend;
@@ -713,8 +792,6 @@ static int route(sim_t* s, int64_t k, int64_t t)
 
     s->i_pre[k] = (uint8_t)ip;
     s->i_dec[k] = (uint8_t)id;
-    s->pre_end[k] = end;
-    s->t_ready[k] = ready;
     return ORC_OK;
 }
 
@@ -740,6 +817,7 @@ static int validate_cfg(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t po
     if (cfg->dec_kv_div < 1 || cfg->pre_base < 1 || cfg->dec_base < 1) return ORC_EINVAL;
     if (cfg->n_classes < 1 || cfg->n_classes > 4) return ORC_EINVAL;
     if (policy < 0 || policy > 4) return ORC_EINVAL;
+    if (cfg->pre_batch_tokens < 0 || cfg->pre_batch_tokens > ((int64_t)1 << 30)) return ORC_EINVAL;
     if (cc->ablate < 0 || cc->ablate > 7) return ORC_EINVAL;
     if (cc->proxy_backlog < 0 || cc->proxy_backlog > 1) return ORC_EINVAL;
     if (cc->poll_us < 0 || cc->poll_us > ARR_LIMIT) return ORC_EINVAL;
@@ -788,14 +866,24 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
     s.inflight = (int64_t*)calloc((size_t)np, 8);
     s.pre_list = (int64_t**)calloc((size_t)np, sizeof(int64_t*));
     s.polled_kv = (int64_t*)calloc((size_t)nd, 8);
+    s.pfifo = (int64_t**)calloc((size_t)np, sizeof(int64_t*));
+    s.prun = (int64_t**)calloc((size_t)np, sizeof(int64_t*));
+    s.pfifo_head = (int64_t*)calloc((size_t)np, 8);
+    s.pfifo_tail = (int64_t*)calloc((size_t)np, 8);
+    s.prun_n = (int64_t*)calloc((size_t)np, 8);
+    s.prun_end = (int64_t*)calloc((size_t)np, 8);
+    s.prun_on = (int64_t*)calloc((size_t)np, 8);
     rc = ORC_OK;
     if (!s.stage || !s.gen || !s.dec_of || !s.admitted || !s.committed || !s.fifo || !s.n_committed ||
         !s.fifo_head || !s.fifo_tail || !s.stepping || !s.steps || !s.busy || !s.inflight || !s.pre_list ||
-        !s.polled_kv)
+        !s.polled_kv || !s.pfifo || !s.prun || !s.pfifo_head || !s.pfifo_tail || !s.prun_n || !s.prun_end ||
+        !s.prun_on)
         rc = ORC_ENOMEM;
     for (int64_t i = 0; i < np && rc == ORC_OK; ++i) {
         s.pre_list[i] = (int64_t*)calloc((size_t)nn, 8);
-        if (!s.pre_list[i]) rc = ORC_ENOMEM;
+        s.pfifo[i] = (int64_t*)calloc((size_t)nn, 8);
+        s.prun[i] = (int64_t*)calloc((size_t)nn, 8);
+        if (!s.pre_list[i] || !s.pfifo[i] || !s.prun[i]) rc = ORC_ENOMEM;
     }
     for (int64_t d = 0; d < nd && rc == ORC_OK; ++d) {
         s.committed[d] = (int64_t*)calloc((size_t)nn, 8);
@@ -819,6 +907,16 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
             st->events += 1;
             if (e.kind == EV_STEP_END) {
                 on_step_end(&s, e.inst, t);
+            } else if (e.kind == EV_PREFILL_END && e.k < 0) {
+                /* a prefill batch ends: all its members leave the instance */
+                int64_t pi = e.inst;
+                for (int64_t m = 0; m < s.prun_n[pi]; ++m) {
+                    int64_t i = 0;
+                    while (s.pre_list[pi][i] != s.prun[pi][m]) ++i;
+                    s.pre_list[pi][i] = s.pre_list[pi][--s.inflight[pi]];
+                }
+                s.prun_n[pi] = 0;
+                s.prun_on[pi] = 0;
             } else if (e.kind == EV_PREFILL_END) {
                 int64_t i = 0;
                 while (s.pre_list[e.inst][i] != e.k) ++i;
@@ -833,9 +931,12 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
             }
         }
         if (rc) break;
-        /* (2) admissions and step starts on every decode instance not mid-step */
+        /* (2) admissions and step starts on every decode instance not mid-step,
+         * and the next batch on every idle prefill instance with a queue */
         for (int64_t d = 0; d < nd && rc == ORC_OK; ++d)
             if (!s.stepping[d]) rc = admit_and_start(&s, d, t);
+        for (int64_t i = 0; i < np && rc == ORC_OK && cfg->pre_batch_tokens > 0; ++i)
+            if (!s.prun_on[i] && s.pfifo_head[i] < s.pfifo_tail[i]) rc = start_prefill_batch(&s, i, t);
         if (rc) break;
         /* the occupancy poll at t sees the state after every event at t and
          * before the arrivals at t [reading: equal-time order] */
@@ -857,9 +958,14 @@ int orc_simulate(const orc_sim_cfg* cfg, const orc_consts* cc, int64_t policy, i
     }
     free(s.stage); free(s.gen); free(s.dec_of); free(s.admitted); free(s.committed); free(s.fifo);
     free(s.n_committed); free(s.fifo_head); free(s.fifo_tail); free(s.stepping); free(s.steps);
-    for (int64_t i = 0; i < np; ++i)
+    for (int64_t i = 0; i < np; ++i) {
         if (s.pre_list) free(s.pre_list[i]);
+        if (s.pfifo) free(s.pfifo[i]);
+        if (s.prun) free(s.prun[i]);
+    }
     free(s.busy); free(s.inflight); free(s.pre_list); free(s.polled_kv); free(s.heap.a);
+    free(s.pfifo); free(s.prun); free(s.pfifo_head); free(s.pfifo_tail); free(s.prun_n); free(s.prun_end);
+    free(s.prun_on);
     return rc;
 }
 

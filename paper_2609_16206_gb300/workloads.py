@@ -23,6 +23,7 @@ LN_16 = float.fromhex("0x1.62e42fefa39efp+1")
 LN_128 = float.fromhex("0x1.3687a9f1af2b1p+2")
 LN_512 = float.fromhex("0x1.8f40b5ed9812dp+2")
 LN_1024 = float.fromhex("0x1.bb9d3beb8c86bp+2")
+LN_2048 = float.fromhex("0x1.e7f9c1e980fa9p+2")
 
 POLICY_LEARNED, POLICY_RR, POLICY_JSQ, POLICY_HEURISTIC, POLICY_LEARNED_P2 = 0, 1, 2, 3, 4
 POLICY_NAMES = {POLICY_LEARNED: "learned", POLICY_RR: "round_robin", POLICY_JSQ: "least_loaded",
@@ -87,6 +88,7 @@ class SimCfg:
     cap_active: int = 1024
     cap_prefill_ring: int = 1024
     heuristic_threshold_tokens: int = 512
+    prefill_batch_tokens: int = 0         # 0: serial FCFS prefill; > 0: batched prefill, token budget per batch
 
     def replace(self, **kw) -> "SimCfg":
         return dataclasses.replace(self, **kw)
@@ -136,6 +138,37 @@ def replica_sweep(n_replicas: int = 4096, n_req: int = 20_000) -> SweepWorkload:
     sc = SimCfg(n_prefill=2, n_decode=6)
     return SweepWorkload(f"replica_sweep_2p6d_{n_replicas}x{n_req}_mmpp", tc, sc,
                          n_replicas=n_replicas, n_req=n_req)
+
+
+U32_ALL = 1 << 32                    # a threshold every 32-bit word is below
+PREFILL_BATCH_TOKENS = 8192          # token budget of one prefill batch in the batched-prefill presets
+
+
+def chat(n_replicas: int = 256, n_req: int = 10_000, rate_mreq: int = 9_000) -> SweepWorkload:
+    """Table 1 'chat' (short in, short out): the single-replica prompt law, every
+    output from the short component; 2P+6D, Poisson."""
+    tc = TraceCfg(rate_mreq=(rate_mreq, rate_mreq), mix_short_thr=U32_ALL)
+    return SweepWorkload(f"chat_2p6d_{n_replicas}x{n_req}", tc, SimCfg(n_prefill=2, n_decode=6),
+                         n_replicas=n_replicas, n_req=n_req)
+
+
+def reasoning(n_replicas: int = 256, n_req: int = 10_000, rate_mreq: int = 4_000) -> SweepWorkload:
+    """Table 1 'reasoning' (short in, long out): every output from the long component."""
+    tc = TraceCfg(rate_mreq=(rate_mreq, rate_mreq), mix_short_thr=0)
+    return SweepWorkload(f"reasoning_2p6d_{n_replicas}x{n_req}", tc, SimCfg(n_prefill=2, n_decode=6),
+                         n_replicas=n_replicas, n_req=n_req)
+
+
+def document(n_replicas: int = 256, n_req: int = 10_000, rate_mreq: int = 5_000,
+             batch_tokens: int = PREFILL_BATCH_TOKENS) -> SweepWorkload:
+    """Table 1 'document' (up to 4k in, short out; stresses prefill compute and
+    KV transfer): prompts lognormal around 2,048 tokens clipped to [16, 4096],
+    outputs from the short component, 2P+6D, Poisson, batched prefill with a
+    `batch_tokens` budget (0 = serial prefill)."""
+    tc = TraceCfg(rate_mreq=(rate_mreq, rate_mreq), prompt_mu=LN_2048, prompt_sigma=0.5, prompt_max=4096,
+                  mix_short_thr=U32_ALL)
+    sc = SimCfg(n_prefill=2, n_decode=6, prefill_batch_tokens=batch_tokens)
+    return SweepWorkload(f"document_2p6d_{n_replicas}x{n_req}", tc, sc, n_replicas=n_replicas, n_req=n_req)
 
 
 def large_pool(n_replicas: int = 16384, n_req: int = 50_000, rate_mreq: int = 33_000) -> SweepWorkload:
