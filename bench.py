@@ -383,7 +383,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "f64f9a4e5f70184c": {"warp_inst": 189399495450, "dram_bytes": 35.78e9 + 25.13e9},
+    "46f931c467a24d1d": {"warp_inst": 188356272513, "dram_bytes": 35.80e9 + 25.11e9},
 }
 
 

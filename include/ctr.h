@@ -97,7 +97,16 @@ typedef struct ctr_trace_cfg {
 
 /* Simulated cluster (a host struct): explicit prefill and decode pools, KV
  * transfer, continuous decode batching with KV reservation, SLO classes, and
- * the capacities of the per-instance structures the GPU keeps. */
+ * the capacities of the per-instance structures the GPU keeps.
+ * Prefill is serial FCFS per instance (prefill_batch_tokens = 0) or batched
+ * (sec. VI implements continuous batching in both stages): an instance runs
+ * one batch at a time, taking FCFS the head of its queue and then every next
+ * request while the batch's prompt tokens stay <= prefill_batch_tokens; a
+ * batch lasts pre_base + pre_per_tok * (its prompt tokens), every member's KV
+ * transfer starts at its end, and a batch starts when the previous one ends
+ * (before arrivals at that instant are routed) or when a request reaches an
+ * idle instance.  The learned router's true prefill backlog is then the rest
+ * of the running batch plus the queue cut into batches by the same rule. */
 typedef struct ctr_sim_cfg {
     int32_t n_prefill, n_decode;      /* >= 1 each, n_prefill + n_decode <= 32 */
     int64_t kv_cap_tokens;            /* C per decode instance, 1..2^31-1 */
@@ -116,6 +125,7 @@ typedef struct ctr_sim_cfg {
     int32_t cap_waiting;              /* KV-ready requests not yet admitted, 1..2^20 */
     int32_t cap_active;               /* decode batch size, 1..2^20 */
     int32_t cap_prefill_ring;         /* requests in flight on a prefill instance, 1..2^20 */
+    int64_t prefill_batch_tokens;     /* 0: serial FCFS prefill; 1..2^30: batched prefill (below) */
 } ctr_sim_cfg;
 
 /* Fixed-point constants of the learned router (a host struct).  Weights carry

@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 3;
+constexpr int kAbiVersion = 4;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -37,6 +37,7 @@ bool valid_sim_cfg(const ctr_sim_cfg* c)
     for (int i = 0; i < CTR_MAX_CLASSES; ++i)
         if (c->ttft_slo_us[i] < 0 || c->tpot_slo_us[i] < 0) return false;
     if (c->max_steps_per_instance < 1) return false;
+    if (!in_range(c->prefill_batch_tokens, 0, 1LL << 30)) return false;
     const int64_t cap_max = 1LL << 20;
     if (!in_range(c->cap_pending, 1, cap_max) || !in_range(c->cap_waiting, 1, cap_max) ||
         !in_range(c->cap_active, 1, cap_max) || !in_range(c->cap_prefill_ring, 1, cap_max))
@@ -213,6 +214,7 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     p.dec_base = cfg->dec_base_us;
     p.dec_seq = cfg->dec_us_per_seq;
     p.kv_div = cfg->dec_kv_tokens_per_us;
+    p.pre_batch = cfg->prefill_batch_tokens;
     // ceil(2^64 / kv_div) = floor((2^64 - 1) / kv_div) + 1 for kv_div >= 2 (not a power of two
     // or otherwise: the +1 rounds up whenever kv_div does not divide 2^64 exactly)
     if (p.kv_div >= 2) {

@@ -74,6 +74,7 @@ struct SimParams {
     int64_t pre_base, pre_tok, xfer_tok;
     int64_t dec_base, dec_seq;
     int64_t kv_div;
+    int64_t pre_batch;          // prefill batch token budget, 0 = serial prefill
     uint64_t kv_div_magic;      // ceil(2^64 / kv_div) (kv_div >= 2)
     int32_t n_classes, heur_thresh;
     int64_t max_steps;

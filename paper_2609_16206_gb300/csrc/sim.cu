@@ -41,6 +41,7 @@ constexpr int64_t kPressureClamp = int64_t(1) << 18;
 constexpr int kRecipN = 1024;  // batch sizes with a tabulated reciprocal
 constexpr int kRingPBits = 21;  // prefill ring entry: end << 21 | p (p <= 2^20)
 constexpr int64_t kRingPMask = (int64_t(1) << kRingPBits) - 1;
+constexpr int kRingKShift = 26;  // batched prefill ring entry: k << 26 | d << 21 | p
 
 // floor((2^64 - 1) / n) for n = 1..kRecipN, for the decode backlog's division
 // by the batch size (built at compile time, read through the read-only path)
@@ -325,10 +326,18 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // workload have the same number of requests, so the groups walk their
 // arrivals in lockstep (request k of every row at once, each at its own time);
 // the per-lane event loops, the per-group argmins and the commits are
-// independent across groups.  kSignals compiles in the deployed proxy's
-// signals (ledger backlog, polled occupancy); the host launches that
-// instantiation only when some constant set asks for one of them.
-template <int G, bool kSignals>
+// independent across groups.  kExt compiles in the deployed proxy's
+// signals (ledger backlog, polled occupancy) and batched prefill; the host
+// launches that instantiation only when a launch asks for one of them.
+//
+// Batched prefill: a prefill lane's ring holds its in-flight requests as
+// k << 26 | d << 21 | p (running batch first, then the queue).  Before the
+// decode lanes advance to an arrival, the prefill lanes end every batch that
+// ends by then and start the next at that instant; each newly started batch
+// (contiguous at the ring's head) is published to the group, and every
+// decode lane copies its own members, now with known KV-ready times, into its
+// pending heap.  Repeated until no prefill lane has another batch ending.
+template <int G, bool kExt>
 __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __grid_constant__ SimParams P)
 {
     constexpr int kRowsPerWarp = 32 / G;
@@ -385,6 +394,71 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
         int32_t rr_p = 0, rr_d = 0;
         uint64_t h = 0;
         int err = CTR_OK;
+        // batched prefill lanes: busy = end of the running batch of run_n members (run_p tokens); the
+        // queue behind it, cut FCFS into budget-limited batches, forms q_batches, the last of q_tail tokens
+        int32_t run_n = 0, q_batches = 0;
+        int64_t run_p = 0, q_tail = 0;
+        const bool batched = kExt && P.pre_batch > 0;
+
+        // Batched prefill: end every batch that ends by T, start the next at that
+        // instant, and hand the members' KV-ready times to their decode lanes
+        // (warp-collective: every lane of the warp calls it).
+        auto prefill_batches = [&](int64_t T) {
+            for (;;) {
+                int32_t pub_n = 0, pub_head = 0;
+                int64_t pub_end = 0;
+                if (live && err == CTR_OK && is_pre && run_n > 0 && busy <= T) {
+                    ring_head += run_n;
+                    if (ring_head >= P.cap_ring) ring_head -= P.cap_ring;
+                    ring_n -= run_n;
+                    ring_sum_p -= run_p;
+                    run_n = 0;
+                    run_p = 0;
+                    if (ring_n > 0) {  // the next batch: the head, then FCFS while the budget holds
+                        int pos = ring_head;
+                        int64_t pmax = 0;
+                        while (run_n < ring_n) {
+                            const int64_t pj = ring[pos * kWarp] & kRingPMask;
+                            if (run_n > 0 && run_p + pj > P.pre_batch) break;
+                            run_p += pj;
+                            pmax = pj > pmax ? pj : pmax;
+                            run_n += 1;
+                            pos = pos + 1 == P.cap_ring ? 0 : pos + 1;
+                        }
+                        busy += P.pre_base + P.pre_tok * run_p;
+                        q_batches -= 1;
+                        if (q_batches == 0) q_tail = 0;
+                        if (busy + P.xfer_tok * pmax >= kTimeLimit) {
+                            err = CTR_EOVERFLOW;
+                        } else {
+                            pub_n = run_n;
+                            pub_head = ring_head;
+                            pub_end = busy;
+                        }
+                    }
+                }
+                if (!__any_sync(kFull, pub_n > 0)) break;
+                const int64_t* const rings = reinterpret_cast<const int64_t*>(sb);
+                for (int i = 0; i < P.n_pre; ++i) {
+                    const int src = grp * G + i;
+                    const int32_t m_i = __shfl_sync(kFull, pub_n, src);
+                    const int32_t h_i = __shfl_sync(kFull, pub_head, src);
+                    const int64_t e_i = __shfl_sync(kFull, pub_end, src);
+                    if (is_dec && live) {
+                        int pos = h_i;
+                        for (int32_t m = 0; m < m_i; ++m) {
+                            const int64_t v = rings[pos * kWarp + src];
+                            if ((int)((v >> kRingPBits) & 31) == gl - P.n_pre) {
+                                const int64_t ready = e_i + P.xfer_tok * (v & kRingPMask);
+                                heap_push(pend, s.pend_n, s.pend_top,
+                                          ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift));
+                            }
+                            pos = pos + 1 == P.cap_ring ? 0 : pos + 1;
+                        }
+                    }
+                }
+            }
+        };
 
         for (int64_t base = 0; base < n; base += G) {
             if (!__any_sync(kFull, live)) break;
@@ -410,9 +484,12 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                 const int64_t ohk = __shfl_sync(kFull, my_oh, j, G);
 
                 // 1. advance every instance to the arrival time
+                if constexpr (kExt) {
+                    if (batched) prefill_batches(T);
+                }
                 if (live) {
                     if (is_dec) {
-                        if (kSignals && cc.poll_us > 0) {
+                        if (kExt && cc.poll_us > 0) {
                             // the router sees the occupancy of the last poll instant floor(T / D) D,
                             // taken after every event at that instant: advance there first
                             const int64_t tp = (int64_t)div_recip((uint64_t)T, (uint64_t)cc.poll_us, cc.poll_recip) *
@@ -424,10 +501,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                             }
                         }
                         if (err == CTR_OK) err = decode_advance(s, T, P, pend, act, wait, tb, ob);
-                    } else if (is_pre) {
+                    } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
                         while (ring_n > 0 && ring_front <= thr) {
-                            if constexpr (kSignals) ring_sum_p -= ring_front & kRingPMask;
+                            if constexpr (kExt) ring_sum_p -= ring_front & kRingPMask;
                             ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
                             ring_n -= 1;
                             ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
@@ -447,7 +524,12 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                     if (is_pre) {
                         if (learned) {
                             int64_t b = busy > T ? busy - T : 0;
-                            if (kSignals && cc.proxy) {  // the ledger: tau_pre0 + tau_pre p per prefill not yet ended
+                            if (batched) {  // the running batch's rest, then the queue's batches
+                                b = (run_n > 0 && busy > T ? busy - T : 0) + P.pre_base * (int64_t)q_batches +
+                                    P.pre_tok * (ring_sum_p - run_p);
+                                if (b > kBacklogClamp) b = kBacklogClamp;
+                            }
+                            if (kExt && cc.proxy) {  // the ledger: tau_pre0 + tau_pre p per prefill not yet ended
                                 b = cc.tau_pre0 * (int64_t)ring_n + cc.tau_pre * ring_sum_p;
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
@@ -471,11 +553,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                                                                       : lo / nd);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            if (kSignals && cc.proxy) {  // the ledger: tau_dec o_hat per request routed here and not done
+                            if (kExt && cc.proxy) {  // the ledger: tau_dec o_hat per request routed here and not done
                                 b = (cc.ablate & CTR_ABLATE_PREDICTED_LENGTH) ? 0 : cc.tau_dec * s.ohat;
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            const int64_t kv = kSignals && cc.poll_us > 0 ? kv_seen : s.kv_res;
+                            const int64_t kv = kExt && cc.poll_us > 0 ? kv_seen : s.kv_res;
                             int64_t press = (int64_t)div_recip((uint64_t)(kv + pk + oh_f) << 16,
                                                                (uint64_t)P.kv_cap, P.kv_cap_recip);
                             if (press > kPressureClamp) press = kPressureClamp;
@@ -521,7 +603,33 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
 
                 // 3. commit: FCFS prefill, KV transfer, queue at the decode instance
                 int64_t ready = 0;
-                if (live && gl == ip) {
+                if (batched && live && gl == ip) {
+                    if (ring_n == P.cap_ring) {
+                        err = CTR_EOVERFLOW;
+                        ready = kTimeLimit;
+                    } else {
+                        int pos = ring_head + ring_n;
+                        if (pos >= P.cap_ring) pos -= P.cap_ring;
+                        ring[pos * kWarp] = (k << kRingKShift) | ((int64_t)id << kRingPBits) | pk;
+                        ring_n += 1;
+                        ring_sum_p += pk;
+                        if (run_n == 0) {  // an idle instance starts a batch of this request at once
+                            busy = T + P.pre_base + P.pre_tok * pk;
+                            run_n = 1;
+                            run_p = pk;
+                            ready = busy + P.xfer_tok * pk;
+                            if (ready >= kTimeLimit) err = CTR_EOVERFLOW;
+                        } else {  // queued: its KV-ready time is known when its batch starts
+                            if (q_batches > 0 && q_tail + pk <= P.pre_batch) {
+                                q_tail += pk;
+                            } else {
+                                q_batches += 1;
+                                q_tail = pk;
+                            }
+                            ready = -1;
+                        }
+                    }
+                } else if (live && gl == ip) {
                     const int64_t start = busy > T ? busy : T;
                     const int64_t end = start + P.pre_base + P.pre_tok * pk;
                     ready = end + P.xfer_tok * pk;
@@ -537,15 +645,15 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                         ring[pos * kWarp] = e;
                         if (ring_n == 0) ring_front = e;
                         ring_n += 1;
-                        if constexpr (kSignals) ring_sum_p += pk;
+                        if constexpr (kExt) ring_sum_p += pk;
                     }
                 }
                 ready = __shfl_sync(kFull, ready, ip, G);
                 if (live && gl == P.n_pre + id && ready < kTimeLimit) {
-                    if (s.pend_n == P.cap_pend) {
+                    if (s.q - s.w_n - s.n_act == P.cap_pend) {  // routed here with KV not yet ready
                         err = CTR_EOVERFLOW;
                     } else {
-                        heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
+                        if (ready >= 0) heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
                         s.q += 1;
                         s.R += ok;
                         s.ohat += ohk;
@@ -562,7 +670,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __gri
                 if (P.i_dec) P.i_dec[ob + kl] = (uint8_t)(my_route & 0xFF);
             }
         }
-        // drain: every remaining event
+        // drain: every remaining batch, then every remaining event
+        if constexpr (kExt) {
+            if (batched) {
+                prefill_batches(kNever - 1);
+                if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
+            }
+        }
         if (live && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob);
 
 #pragma unroll
@@ -653,6 +767,7 @@ cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cuda
     (void)warps_per_block;
     bool signals = false;
     for (int i = 0; i < p.n_sets; ++i) signals = signals || p.sets[i].proxy != 0 || p.sets[i].poll_us > 0;
+    signals = signals || p.pre_batch > 0;
     const dim3 grid(blocks), block(kWarpsPerBlock * 32);
     switch (sim_group_width(p.n_pre + p.n_dec) * 2 + (signals ? 1 : 0)) {
     case 8: sim_kernel<4, false><<<grid, block, 0, stream>>>(p); break;

@@ -60,7 +60,7 @@ class CtrSimCfg(C.Structure):
                 ("ttft_slo_us", C.c_int64 * 4), ("tpot_slo_us", C.c_int64 * 4),
                 ("max_steps_per_instance", C.c_int64),
                 ("cap_pending", C.c_int32), ("cap_waiting", C.c_int32), ("cap_active", C.c_int32),
-                ("cap_prefill_ring", C.c_int32)]
+                ("cap_prefill_ring", C.c_int32), ("prefill_batch_tokens", C.c_int64)]
 
 
 class CtrCostConsts(C.Structure):
@@ -169,6 +169,7 @@ def sim_cfg_struct(sc) -> CtrSimCfg:
     s.max_steps_per_instance = int(sc.max_steps_per_instance)
     s.cap_pending, s.cap_waiting = int(sc.cap_pending), int(sc.cap_waiting)
     s.cap_active, s.cap_prefill_ring = int(sc.cap_active), int(sc.cap_prefill_ring)
+    s.prefill_batch_tokens = int(getattr(sc, "prefill_batch_tokens", 0))
     return s
 
 

@@ -36,7 +36,7 @@ def test_exports_every_declared_function(libctr):
 def test_static_entry_points_run_without_gpu(libctr):
     libctr.ctr_strerror.restype = ctypes.c_char_p
     assert libctr.ctr_strerror(-3).decode().startswith("a fixed-capacity")
-    assert libctr.ctr_abi_version() == 3
+    assert libctr.ctr_abi_version() == 4
 
 
 def test_struct_layout_matches_header(tmp_path):

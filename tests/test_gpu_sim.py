@@ -256,3 +256,57 @@ def test_proxy_signals_host_validation():
     for bad in (dict(proxy_backlog=2), dict(poll_us=-1), dict(poll_us=(1 << 39) + 1)):
         with pytest.raises(ctr.CtrError):
             simulate(ctr, wl.sim, [W.CALIBRATED.replace(**bad)], [W.POLICY_LEARNED], tr, 1, 16)
+
+
+ALL_FIVE = [W.POLICY_LEARNED, W.POLICY_RR, W.POLICY_JSQ, W.POLICY_HEURISTIC, W.POLICY_LEARNED_P2]
+
+
+@pytest.mark.parametrize("budget", [900, 8192, 1 << 20])
+def test_batched_prefill_document(orc, budget):
+    """Batched prefill (sec. VI) on the Table 1 document workload, every policy."""
+    ctr = need_gpu()
+    wl = W.document(rate_mreq=6_500, batch_tokens=budget)
+    R, N = 3, 2000
+    tr = gen(ctr, wl.trace, R, N)
+    res = simulate(ctr, wl.sim, [W.CALIBRATED], ALL_FIVE, tr, R, N)
+    _check_rows(orc, wl.sim, [W.CALIBRATED], ALL_FIVE, [host_trace(tr, r) for r in range(R)], res, N)
+
+
+def test_batched_prefill_equal_times(orc):
+    """Arrivals on a 10 ms grid and batches of constant length 20 ms: arrivals
+    land on batch ends all the time (the batch that starts there must not take
+    them), with the proxy signals on as well."""
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    R, N = 3, 2000
+    tr = gen(ctr, wl.trace.replace(rate_mreq=(20_000, 60_000)), R, N)
+    tr["arrival_us"].copy_((tr["arrival_us"] // 10_000) * 10_000)
+    torch.cuda.synchronize()
+    sc = wl.sim.replace(pre_us_per_tok=0, prefill_batch_tokens=3000, n_prefill=3, n_decode=5)
+    sets = [W.CALIBRATED, W.as_deployed(W.CALIBRATED)]
+    res = simulate(ctr, sc, sets, ALL_FIVE, tr, R, N)
+    _check_rows(orc, sc, sets, ALL_FIVE, [host_trace(tr, r) for r in range(R)], res, N)
+
+
+@pytest.mark.parametrize("caps", [dict(cap_prefill_ring=24), dict(cap_pending=12), dict(cap_waiting=2),
+                                  dict(cap_active=20)], ids=lambda c: list(c)[0])
+def test_batched_prefill_capacity_errors(orc, caps):
+    ctr = need_gpu()
+    wl = W.document(rate_mreq=9_000)
+    R, N = 3, 1500
+    tr = gen(ctr, wl.trace, R, N)
+    sc = wl.sim.replace(**caps)
+    res = simulate(ctr, sc, [W.CALIBRATED], ALL_FIVE, tr, R, N)
+    _check_rows(orc, sc, [W.CALIBRATED], ALL_FIVE, [host_trace(tr, r) for r in range(R)], res, N)
+    assert (res["status"] == -3).any()
+
+
+@pytest.mark.parametrize("wl", [W.chat(), W.reasoning(), W.large_pool(rate_mreq=34_000)], ids=["chat", "reasoning", "4p28d"])
+def test_workload_families_batched_prefill(orc, wl):
+    ctr = need_gpu()
+    R, N = 2, 2000
+    tr = gen(ctr, wl.trace, R, N)
+    sc = wl.sim.replace(prefill_batch_tokens=W.PREFILL_BATCH_TOKENS)
+    sets = [wl.consts[0], W.as_deployed(wl.consts[0])]
+    res = simulate(ctr, sc, sets, ALL_FIVE, tr, R, N)
+    _check_rows(orc, sc, sets, ALL_FIVE, [host_trace(tr, r) for r in range(R)], res, N)
