@@ -9,8 +9,10 @@
   crosses 1/2 (the paper drives every workload at the rate where round-robin
   is "mid-collapse", found by probing, sec. IV-B): an integer bisection over
   milli-requests per second, every probe a GPU simulation.
-* ``calibration_sweep`` / ``large_pool_stress`` -- the mispriced-constants x
-  pool-width sweep and the scarcity stress workload built on those rates.
+* ``calibration_sweep_cfgs`` / ``load_rate`` -- the mispriced-constants x
+  pool-width sweep grid and its offered rates.
+* ``noise_sweep`` -- the predictor-noise sweep of sec. V-G: the same replicas
+  at every noise level (common random numbers), one simulation call.
 
 Everything here is argument marshalling and control flow; the arithmetic runs
 in the CUDA kernels behind ``ctr``.
@@ -120,3 +122,24 @@ def calibration_sweep_cfgs(widths=(3, 4, 5, 6, 7), mixes=(1.0, 5 / 6, 2 / 3, 1 /
 def load_rate(sat_mreq: int, load: float) -> int:
     """Offered rate = load x saturation rate, rounded half up, at least 1."""
     return max(1, int(sat_mreq * load + 0.5))
+
+
+NOISE_SIGMAS = (0.0, 0.25, 0.5, 0.75, 1.0, 1.25, 1.5)  # sec. V-G injects up to 150 % relative error
+
+
+def noise_sweep(wl, sigmas=NOISE_SIGMAS, seeds: int = 16, const_sets=None, policies=None, device="cuda"):
+    """Every predictor-noise level in `sigmas` on the same `seeds` replicas of
+    workload `wl` (replica slice [i * seeds, (i + 1) * seeds) has noise
+    sigmas[i]; arrivals, lengths and the noise draws are shared, only the
+    prediction's spread changes), simulated and scored in one call each.
+    Returns (buffers, n_replicas)."""
+    const_sets = const_sets or wl.consts
+    policies = policies or list(W.ALL_POLICIES)
+    R = len(sigmas) * seeds
+    rows = R * len(const_sets) * len(policies)
+    buf = alloc(wl.sim, R, rows, wl.n_req, device)
+    for i, sg in enumerate(sigmas):
+        view = {name: t[i * seeds:(i + 1) * seeds] for name, t in buf.trace.items()}
+        ctr.ctr_gen_trace(wl.trace.replace(noise_sigma=float(sg)), seeds, 0, wl.n_req, view)
+    run_step(None, wl.sim, const_sets, policies, R, wl.n_req, 0, buf, gen=False)
+    return buf, R

@@ -121,3 +121,29 @@ def test_large_pool_stress_reduced(orc):
 def test_large_pool_stress_full_size_sampled(orc):
     """16,384 replicas x 50,000 requests, 4P+28D at 1.2x the saturation rate, all four policies."""
     _large_pool_case(orc, n_replicas=16384, n_req=50_000, sample_replicas=(0, 16383))
+
+
+def test_noise_sweep(orc):
+    """sec. V-G: predictor noise 0..150 % on the same replicas, one launch; sampled rows = oracle, and the
+    learned router's routes depend on the noise while round-robin's do not."""
+    ctr = need_gpu()
+    from paper_2609_16206_gb300 import sweep
+    wl = W.replica_sweep(n_req=2000)
+    seeds = 3
+    buf, R = sweep.noise_sweep(wl, seeds=seeds)
+    torch.cuda.synchronize()
+    h = buf.row_hash.cpu().numpy().astype(np.uint64)
+    st = buf.row_status.cpu().numpy()
+    assert (st == 0).all()
+    n_pol = len(W.ALL_POLICIES)
+    for i, sg in enumerate(sweep.NOISE_SIGMAS):
+        r = i * seeds + 1
+        trh = host_trace(buf.trace, r)
+        ref = orc.gen_trace(wl.trace.replace(noise_sigma=sg), wl.n_req, replica=1)
+        for key in ref:
+            assert np.array_equal(trh[key], ref[key]), key
+        for j, pol in enumerate(W.ALL_POLICIES):
+            assert int(h[r * n_pol + j]) == orc.simulate(wl.sim, W.CALIBRATED, pol, trh)["hash"]
+    rr = [int(h[(i * seeds) * n_pol + 1]) for i in range(len(sweep.NOISE_SIGMAS))]
+    lr = [int(h[(i * seeds) * n_pol + 0]) for i in range(len(sweep.NOISE_SIGMAS))]
+    assert len(set(rr)) == 1 and len(set(lr)) == len(lr)
