@@ -383,7 +383,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "46f931c467a24d1d": {"warp_inst": 188356272513, "dram_bytes": 35.80e9 + 25.11e9},
+    "35e9cb07164055b9": {"warp_inst": 184138909465, "dram_bytes": 32.57e9 + 22.29e9},
 }
 
 

@@ -337,8 +337,8 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // (contiguous at the ring's head) is published to the group, and every
 // decode lane copies its own members, now with known KV-ready times, into its
 // pending heap.  Repeated until no prefill lane has another batch ending.
-template <int G, bool kExt>
-__global__ void __launch_bounds__(kWarpsPerBlock * 32, 8) sim_kernel(const __grid_constant__ SimParams P)
+template <int G, bool kExt, int kBlocksPerSM>
+__global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(const __grid_constant__ SimParams P)
 {
     constexpr int kRowsPerWarp = 32 / G;
     const int lane = threadIdx.x & 31;
@@ -746,12 +746,13 @@ int sim_max_resident_warps(int* warps_per_block, int* blocks)
     int dev = 0, sms = 0, per_sm = 0, per_sm_g = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    // the smallest occupancy over the group widths, so one workspace size fits every launch
+    // the smallest occupancy over the group widths at 8 blocks per SM, so one
+    // workspace size fits every launch
     per_sm = 1 << 30;
-    const void* kernels[8] = {(const void*)sim_kernel<4, false>, (const void*)sim_kernel<8, false>,
-                              (const void*)sim_kernel<16, false>, (const void*)sim_kernel<32, false>,
-                              (const void*)sim_kernel<4, true>, (const void*)sim_kernel<8, true>,
-                              (const void*)sim_kernel<16, true>, (const void*)sim_kernel<32, true>};
+    const void* kernels[8] = {(const void*)sim_kernel<4, false, 8>, (const void*)sim_kernel<8, false, 8>,
+                              (const void*)sim_kernel<16, false, 8>, (const void*)sim_kernel<32, false, 8>,
+                              (const void*)sim_kernel<4, true, 8>, (const void*)sim_kernel<8, true, 8>,
+                              (const void*)sim_kernel<16, true, 8>, (const void*)sim_kernel<32, true, 8>};
     for (const void* k : kernels) {
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_g, k, kWarpsPerBlock * 32, 0) != cudaSuccess)
             return 0;
@@ -762,23 +763,47 @@ int sim_max_resident_warps(int* warps_per_block, int* blocks)
     return sms * per_sm * kWarpsPerBlock;
 }
 
+namespace {
+
+// 7 blocks per SM (72 registers a thread, fewer spills) when all of the
+// launch's persistent warps fit on the GPU at that occupancy -- the common
+// case of one row group per warp -- else 8 (more warps to hide latency).
+template <int G, bool kExt>
+cudaError_t launch_width(const SimParams& p, int blocks, cudaStream_t stream)
+{
+    int dev = 0, sms = 0, per_sm7 = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return cudaErrorInvalidDevice;
+    cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm7, sim_kernel<G, kExt, 7>, kWarpsPerBlock * 32, 0);
+    if (e != cudaSuccess) return e;
+    if ((int64_t)p.n_slots <= (int64_t)sms * per_sm7 * kWarpsPerBlock)
+        sim_kernel<G, kExt, 7><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
+    else
+        sim_kernel<G, kExt, 8><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
 cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
 {
     (void)warps_per_block;
-    bool signals = false;
-    for (int i = 0; i < p.n_sets; ++i) signals = signals || p.sets[i].proxy != 0 || p.sets[i].poll_us > 0;
-    signals = signals || p.pre_batch > 0;
-    const dim3 grid(blocks), block(kWarpsPerBlock * 32);
-    switch (sim_group_width(p.n_pre + p.n_dec) * 2 + (signals ? 1 : 0)) {
-    case 8: sim_kernel<4, false><<<grid, block, 0, stream>>>(p); break;
-    case 9: sim_kernel<4, true><<<grid, block, 0, stream>>>(p); break;
-    case 16: sim_kernel<8, false><<<grid, block, 0, stream>>>(p); break;
-    case 17: sim_kernel<8, true><<<grid, block, 0, stream>>>(p); break;
-    case 32: sim_kernel<16, false><<<grid, block, 0, stream>>>(p); break;
-    case 33: sim_kernel<16, true><<<grid, block, 0, stream>>>(p); break;
-    case 64: sim_kernel<32, false><<<grid, block, 0, stream>>>(p); break;
-    default: sim_kernel<32, true><<<grid, block, 0, stream>>>(p); break;
+    bool ext = false;  // the proxy's signals or batched prefill
+    for (int i = 0; i < p.n_sets; ++i) ext = ext || p.sets[i].proxy != 0 || p.sets[i].poll_us > 0;
+    ext = ext || p.pre_batch > 0;
+    cudaError_t e;
+    switch (sim_group_width(p.n_pre + p.n_dec) * 2 + (ext ? 1 : 0)) {
+    case 8: e = launch_width<4, false>(p, blocks, stream); break;
+    case 9: e = launch_width<4, true>(p, blocks, stream); break;
+    case 16: e = launch_width<8, false>(p, blocks, stream); break;
+    case 17: e = launch_width<8, true>(p, blocks, stream); break;
+    case 32: e = launch_width<16, false>(p, blocks, stream); break;
+    case 33: e = launch_width<16, true>(p, blocks, stream); break;
+    case 64: e = launch_width<32, false>(p, blocks, stream); break;
+    default: e = launch_width<32, true>(p, blocks, stream); break;
     }
+    if (e != cudaSuccess) return e;
     if (p.n_rows > 0) {
         const int64_t hb = p.n_rows < (int64_t)blocks * 8 ? p.n_rows : (int64_t)blocks * 8;
         hash_kernel<<<(unsigned)hb, kHashThreads, 0, stream>>>(p);
