@@ -383,7 +383,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "35e9cb07164055b9": {"warp_inst": 184138909465, "dram_bytes": 32.57e9 + 22.29e9},
+    "6a00efdfe2c4a330": {"warp_inst": 166695257562, "dram_bytes": 32.37e9 + 22.33e9},
 }
 
 

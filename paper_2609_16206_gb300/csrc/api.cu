@@ -231,6 +231,7 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     p.cap_wait = cfg->cap_waiting;
     p.cap_act = cfg->cap_active;
     p.cap_ring = cfg->cap_prefill_ring;
+    p.cap_pend_store = cfg->cap_pending + cfg->cap_waiting + 1;
     p.n_sets = n_const_sets;
     p.n_pols = n_policies;
     for (int i = 0; i < n_policies; ++i) p.pols[i] = policy_ids[i];

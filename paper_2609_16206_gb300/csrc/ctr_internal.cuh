@@ -79,6 +79,7 @@ struct SimParams {
     int32_t n_classes, heur_thresh;
     int64_t max_steps;
     int32_t cap_pend, cap_wait, cap_act, cap_ring;
+    int32_t cap_pend_store;     // pending heap entries: cap_pend + cap_wait + 1
     int32_t n_sets, n_pols;
     int32_t pols[8];
     int64_t n_req, n_rows;
@@ -87,7 +88,7 @@ struct SimParams {
     uint32_t* next_row;
     int64_t slot_bytes;
     int64_t off_act, off_wait;  // byte offsets of the active heap and waiting ring inside a slot
-    int32_t cap_pr;             // max(cap_pend, cap_ring): entries of the first region
+    int32_t cap_pr;             // max(cap_pend_store, cap_ring): entries of the first region
     int32_t n_slots;
     ctr_requests trace;
     uint8_t* i_pre;

@@ -170,7 +170,26 @@ struct Decode {
     bool stepping;
 };
 
-// Advance one decode instance through every event at times <= T.
+// Move every pending request whose KV is ready by t into the waiting FIFO, in
+// (time, index) order; the FIFO's size is checked after each insertion.
+__device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams& P, uint64_t* pend, uint32_t* wait)
+{
+    while (s.pend_n > 0 && (int64_t)(s.pend_top >> kKeyBits) <= t) {
+        const uint32_t k = (uint32_t)(s.pend_top & kKeyMask);
+        heap_pop(pend, s.pend_n, s.pend_top);
+        if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
+        int pos = s.w_head + s.w_n;
+        if (pos >= P.cap_wait) pos -= P.cap_wait;
+        wait[pos * kWarp] = k;
+        s.w_n += 1;
+    }
+    return CTR_OK;
+}
+
+// Advance one decode instance through every event at times <= T.  The pending
+// heap may hold requests already KV-ready (taken at the next step end); it has
+// room for cap_pend + cap_wait + 1 entries, so a full heap means the waiting
+// FIFO has overflowed.
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
                                               uint32_t* wait, int64_t tb, int64_t ob)
 {
@@ -205,10 +224,12 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.step_end += m * S;
             if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
         }
-        const int64_t te = s.stepping ? s.step_end : kNever;
-        const int64_t tev = te < tp ? te : tp;
+        // A KV-ready event while a step runs only matters at the step's end (the
+        // next admission), so it is taken there, in the same pass: the next
+        // event is the running step's end, or the next KV-ready when idle.
+        const int64_t tev = s.stepping ? s.step_end : tp;
         if (tev > T) return CTR_OK;
-        if (te == tev) {  // (1) the running step ends: one token for every active request
+        if (s.stepping) {  // (1) the running step ends: one token for every active request
             s.step_idx += 1;
             s.kv_res += s.n_act;
             s.R -= s.n_act;
@@ -227,16 +248,9 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 P.t_done[ob + k] = tev;
             }
         }
-        // (2) KV-ready requests join the waiting FIFO in (time, index) order
-        while (s.pend_n > 0 && (int64_t)(s.pend_top >> kKeyBits) == tev) {
-            const uint32_t k = (uint32_t)(s.pend_top & kKeyMask);
-            heap_pop(pend, s.pend_n, s.pend_top);
-            if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
-            int pos = s.w_head + s.w_n;
-            if (pos >= P.cap_wait) pos -= P.cap_wait;
-            wait[pos * kWarp] = k;
-            s.w_n += 1;
-        }
+        // (2) every request KV-ready by now joins the waiting FIFO in (time, index) order
+        const int rc = flush_ready(s, tev, P, pend, wait);
+        if (rc != CTR_OK) return rc;
         // (3) not mid-step: strict FCFS admission while the reservation fits, then start a step
         if (!s.stepping) {
             const int pos0 = s.w_head;
@@ -450,8 +464,12 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                             const int64_t v = rings[pos * kWarp + src];
                             if ((int)((v >> kRingPBits) & 31) == gl - P.n_pre) {
                                 const int64_t ready = e_i + P.xfer_tok * (v & kRingPMask);
-                                heap_push(pend, s.pend_n, s.pend_top,
-                                          ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift));
+                                if (s.pend_n == P.cap_pend_store) {
+                                    err = CTR_EOVERFLOW;  // the waiting FIFO has overflowed
+                                } else {
+                                    heap_push(pend, s.pend_n, s.pend_top,
+                                              ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift));
+                                }
                             }
                             pos = pos + 1 == P.cap_ring ? 0 : pos + 1;
                         }
@@ -494,7 +512,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                             // taken after every event at that instant: advance there first
                             const int64_t tp = (int64_t)div_recip((uint64_t)T, (uint64_t)cc.poll_us, cc.poll_recip) *
                                                cc.poll_us;
-                            if (tp > last_poll) {
+                            if (err == CTR_OK && tp > last_poll) {
                                 err = decode_advance(s, tp, P, pend, act, wait, tb, ob);
                                 kv_seen = s.kv_res;
                                 last_poll = tp;
@@ -650,7 +668,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 }
                 ready = __shfl_sync(kFull, ready, ip, G);
                 if (live && gl == P.n_pre + id && ready < kTimeLimit) {
-                    if (s.q - s.w_n - s.n_act == P.cap_pend) {  // routed here with KV not yet ready
+                    // requests routed here whose KV is not ready yet, exactly: first move
+                    // those already ready (kept in the heap until the step end) if it matters
+                    if (s.q - s.w_n - s.n_act >= P.cap_pend) err = flush_ready(s, T, P, pend, wait);
+                    if (err != CTR_OK || s.q - s.w_n - s.n_act == P.cap_pend ||
+                        (ready >= 0 && s.pend_n == P.cap_pend_store)) {
                         err = CTR_EOVERFLOW;
                     } else {
                         if (ready >= 0) heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
@@ -726,7 +748,8 @@ __global__ void __launch_bounds__(kHashThreads) hash_kernel(const __grid_constan
 
 int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr)
 {
-    const int64_t pr = cfg.cap_pending > cfg.cap_prefill_ring ? cfg.cap_pending : cfg.cap_prefill_ring;
+    const int64_t pend_store = (int64_t)cfg.cap_pending + cfg.cap_waiting + 1;  // pending heap entries
+    const int64_t pr = pend_store > cfg.cap_prefill_ring ? pend_store : cfg.cap_prefill_ring;
     const int64_t a = pr * 8 * kWarp;
     const int64_t b = a + (int64_t)cfg.cap_active * 8 * kWarp;
     const int64_t c = b + (int64_t)cfg.cap_waiting * 4 * kWarp;
