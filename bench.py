@@ -256,7 +256,6 @@ def run_ours(args, rank, world, local_rank):
     routed_per_step = rows * N * world
     value = routed_per_step / (ms_step / 1e3)
     per_kernel_ms = {k: v / args.steps for k, v in times.items()}
-    pairs_per_s = N_SCORE_REQ * N_SCORE_INST / (per_kernel_ms["score"] / 1e3)
 
     # ---- end to end through the public API with host buffers (rank-local)
     host_tr = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True) for k, v in tr.items()}
@@ -305,24 +304,69 @@ def run_ours(args, rank, world, local_rank):
         torch.distributed.all_reduce(e2e_t, op=torch.distributed.ReduceOp.MAX)
     e2e_value = None if args.no_e2e else routed_per_step / float(e2e_t.item())
 
+    # ---- the 2^20 scorer as its measurement rule asks: 30 buffer sets (534 MB, > 4x L2) launched back to
+    # back from one CUDA graph, so every launch reads its inputs from HBM and launch gaps are not timed
+    rot_sets = 30
+    rot = [[torch.from_numpy(x).to(dev) for x in (p, oh, cls)] +
+           [torch.empty(N_SCORE_REQ, dtype=torch.int32, device=dev),
+            torch.empty(N_SCORE_REQ, dtype=torch.float32, device=dev)] for _ in range(rot_sets)]
+    with torch.cuda.stream(stream):
+        for b in rot:
+            ctr.ctr_score_batch(b[0], b[1], b[2], sQ, sA, skap, W.SCORE_CONSTS, b[3], b[4], stream=stream)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    cap = torch.cuda.Stream(device=dev)  # capture needs a stream of its own; replay runs on `stream`
+    cap.wait_stream(stream)
+    with torch.cuda.graph(graph, stream=cap):
+        for b in rot:
+            ctr.ctr_score_batch(b[0], b[1], b[2], sQ, sA, skap, W.SCORE_CONSTS, b[3], b[4], stream=cap)
+    stream.wait_stream(cap)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    g_reps = 5
+    g0 = torch.cuda.Event(enable_timing=True)
+    g1 = torch.cuda.Event(enable_timing=True)
+    g0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(g_reps):
+            graph.replay()
+    g1.record(stream)
+    torch.cuda.synchronize()
+    rot_ms = g0.elapsed_time(g1) / (g_reps * rot_sets)
+    rot_ok = all(torch.equal(b[3], rot[0][3]) for b in rot[1:])
+    del graph, rot
+
     # ---- the scorer once more on 2^24 requests (285 MB per launch, beyond L2): its HBM roofline
     big_n = 1 << 24
     bp, boh, bcls = W.score_requests(big_n, seed=2)
-    bsp, bsoh, bscls = (torch.from_numpy(x).to(dev) for x in (bp, boh, bcls))
-    bam = torch.empty(big_n, dtype=torch.int32, device=dev)
-    bcost = torch.empty(big_n, dtype=torch.float32, device=dev)
-    for _ in range(3):
-        ctr.ctr_score_batch(bsp, bsoh, bscls, sQ, sA, skap, W.SCORE_CONSTS, bam, bcost, stream=stream)
+    big = [[torch.from_numpy(x).to(dev) for x in (bp, boh, bcls)] +
+           [torch.empty(big_n, dtype=torch.int32, device=dev), torch.empty(big_n, dtype=torch.float32, device=dev)]
+           for _ in range(2)]  # two sets of 285 MB, alternated: each launch reads from HBM
+    with torch.cuda.stream(stream):
+        for b in big:
+            ctr.ctr_score_batch(b[0], b[1], b[2], sQ, sA, skap, W.SCORE_CONSTS, b[3], b[4], stream=stream)
+    torch.cuda.synchronize()
+    reps = 10
+    graph = torch.cuda.CUDAGraph()
+    cap.wait_stream(stream)
+    with torch.cuda.graph(graph, stream=cap):
+        for i in range(reps):
+            b = big[i % 2]
+            ctr.ctr_score_batch(b[0], b[1], b[2], sQ, sA, skap, W.SCORE_CONSTS, b[3], b[4], stream=cap)
+    stream.wait_stream(cap)
+    with torch.cuda.stream(stream):
+        graph.replay()
+    torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    reps = 10
     e0.record(stream)
-    for _ in range(reps):
-        ctr.ctr_score_batch(bsp, bsoh, bscls, sQ, sA, skap, W.SCORE_CONSTS, bam, bcost, stream=stream)
+    with torch.cuda.stream(stream):
+        graph.replay()
     e1.record(stream)
     torch.cuda.synchronize()
     big_ms = e0.elapsed_time(e1) / reps
-    del bsp, bsoh, bscls, bam, bcost
+    del graph, big
 
     if rank != 0:
         return 0
@@ -344,9 +388,13 @@ def run_ours(args, rank, world, local_rank):
         sim_roof["traffic"] = inst.get("dram_bytes")
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     score_bytes = 17 * N_SCORE_REQ + 3 * 4 * N_SCORE_INST
-    score_roof = {"bound": "hbm", "unit": "GB/s", "achieved": score_bytes / (per_kernel_ms["score"] / 1e3) / 1e9,
-                  "peak": hbm, "traffic": 9.50e6,
-                  "traffic_note": "ncu DRAM read 9.50 MB, write 0 B within the launch (outputs stay in L2)"}
+    pairs_per_s = N_SCORE_REQ * N_SCORE_INST / (rot_ms / 1e3)  # graph-batched launches, inputs from HBM
+    score_roof = {"bound": "hbm", "unit": "GB/s", "achieved": score_bytes / (rot_ms / 1e3) / 1e9,
+                  "peak": hbm, "traffic": 9.50e6, "launch_ms": rot_ms, "launch_ms_in_step": per_kernel_ms["score"],
+                  "traffic_note": "ncu DRAM read 9.50 MB, write 0 B within one graph launch (the 8.4 MB of outputs "
+                                  "are written back from L2 after it)",
+                  "timing": f"{rot_sets} buffer sets ({rot_sets * score_bytes / 1e6:.0f} MB, > 4x L2) back to back "
+                            f"from one CUDA graph, x{g_reps}; outputs identical across sets: {rot_ok}"}
     score_roof["frac"] = score_roof["achieved"] / hbm
     big_bytes = 17 * big_n + 3 * 4 * N_SCORE_INST
     score_roof_big = {"bound": "hbm", "unit": "GB/s", "achieved": big_bytes / (big_ms / 1e3) / 1e9, "peak": hbm,
@@ -383,7 +431,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "6a00efdfe2c4a330": {"warp_inst": 166695257562, "dram_bytes": 32.37e9 + 22.33e9},
+    "d3d7298c094004a9": {"warp_inst": 165467741269, "dram_bytes": 32.14e9 + 21.94e9},
 }
 
 

@@ -211,12 +211,16 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             const int64_t n = s.n_act;
             const int64_t q1 = kv_term(s.kv_res + n, P);  // KV term of the next step
             const int64_t S = P.dec_base + P.dec_seq * n + q1;
+            // plain end j happens at step_end + (j - 1) S <= limit (usually the binding bound)
+            int64_t m = m_fin;
+            const int64_t span = limit - s.step_end;
+            if ((m_fin - 1) * S > span) {  // then span < 2^20 * 2^37
+                m = (span < (int64_t(1) << 56) ? floor_div_small(span, S) : span / S) + 1;
+            }
             const int64_t room = (q1 + 1) * P.kv_div - 1 - s.kv_res;  // the term stays q1 while j n <= room
-            const int64_t m_kv = n <= kRecipN ? (int64_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n]))
-                                              : room / n;
-            int64_t m = m_fin < m_kv ? m_fin : m_kv;
-            const int64_t span = limit - s.step_end;  // plain end j happens at step_end + (j - 1) S <= limit
-            if ((m - 1) * S > span) m = floor_div_small(span, S) + 1;
+            if (m * n > room) {  // the KV term changes first: m = floor(room / n) >= 1
+                m = n <= kRecipN ? (int64_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n])) : room / n;
+            }
             s.step_idx += m;
             s.kv_res += m * n;
             s.R -= m * n;
@@ -532,6 +536,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 }
                 if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
 
+                __syncwarp();  // the lanes leave their event loops at different passes: regroup
                 // 2. price the candidates and take the argmin of each pool
                 uint64_t cost = kEmpty;
                 if (live && pol != CTR_POLICY_ROUND_ROBIN) {
