@@ -16,6 +16,7 @@ times the CPU oracle (the only reference this method has) on the host cores.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import multiprocessing as mp
@@ -435,6 +436,89 @@ SIM_INST_PER_LAUNCH: dict = {
 }
 
 
+WORKLOADS = ("replica_sweep", "single_replica", "large_pool", "calibration_sweep", "document")
+
+
+def run_workload(args):
+    """The other workload shapes (single GPU): trace generation, simulation under
+    every policy and goodput per step, timed like the default workload; one
+    JSON line.  For the record of their throughput beside the benchmarked
+    sweep; the default run never takes this path."""
+    import torch
+
+    from paper_2609_16206_gb300 import build as ctr_build
+    ctr_build.build()
+    from paper_2609_16206_gb300 import ctr, sweep
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    name = args.workload
+    info = {}
+    if name == "calibration_sweep":
+        t_sat = time.perf_counter()
+        sat = sweep.calibration_saturation()
+        torch.cuda.synchronize()
+        info["saturation_search_s"] = time.perf_counter() - t_sat
+        n_sets = len(W.mispriced_sets())
+        routed = 5 * 4 * 4 * 16 * (n_sets + 3) * 10_000
+        cfg = {"workload": "calibration_sweep_2p3d-2p7d_256seeds_x10000", "widths": "3-7 decode (2P)",
+               "replicas_per_width": 256, "learned_sets": n_sets, "baselines": 3,
+               "loads": "0.8 / 0.967 / 1.133 / 1.3 x saturation", "mixes": "100/83/67/50 % short"}
+        state = {}
+
+        def step():
+            state["out"] = sweep.calibration_sweep(sat)
+    else:
+        if name == "single_replica":
+            wl = W.single_replica()
+        elif name == "document":
+            wl = W.document(n_replicas=args.replicas or 4096, n_req=args.requests or 10_000)
+        elif name == "large_pool":
+            base = W.large_pool(n_replicas=args.replicas or 16384, n_req=args.requests or 50_000)
+            t_sat = time.perf_counter()
+            sat = sweep.saturation_rate([base.trace], base.sim, n_req=10_000)[0]
+            info["saturation_search_s"] = time.perf_counter() - t_sat
+            info["rate_mreq"] = sweep.load_rate(sat, 1.2)
+            wl = dataclasses.replace(base, trace=base.trace.replace(rate_mreq=(info["rate_mreq"],) * 2))
+        else:
+            wl = W.replica_sweep(n_replicas=args.replicas or 4096, n_req=args.requests or 20_000)
+        pols = list(W.ALL_POLICIES)
+        rows = wl.n_replicas * len(wl.consts) * len(pols)
+        routed = rows * wl.n_req
+        buf = sweep.alloc(wl.sim, wl.n_replicas, rows, wl.n_req, dev)
+        cfg = {"workload": wl.name, "replicas": wl.n_replicas, "requests_per_replica": wl.n_req,
+               "pool": f"{wl.sim.n_prefill}P+{wl.sim.n_decode}D", "policies": len(pols),
+               "prefill_batch_tokens": wl.sim.prefill_batch_tokens}
+
+        def step():
+            sweep.run_step(wl.trace, wl.sim, wl.consts, pols, wl.n_replicas, wl.n_req, 0, buf, stream=stream)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(0)
+    clocks.start()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms_step = t0.elapsed_time(t1) / args.steps
+    if name == "calibration_sweep":
+        failed = sum(int((b.row_status != 0).sum()) for pair in state["out"].values() for b in pair)
+    else:
+        failed = int((buf.row_status != 0).sum())
+    cfg.update(info)
+    print(json.dumps({
+        "metric": "routed requests/sec", "value": routed / (ms_step / 1e3), "unit": "routed requests/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
+        "higher_is_better": True, "dtype": "int64", "data": "synthetic", "config": cfg,
+        "rows_failed": failed, "note": "trace generation + simulation + goodput per step", "clocks": clk}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -446,12 +530,18 @@ def main():
     ap.add_argument("--replicas", type=int, default=None,
                     help="replicas per GPU (profiling a smaller case; default: the benchmarked 4,096)")
     ap.add_argument("--requests", type=int, default=None, help="requests per replica (default 20,000)")
+    ap.add_argument("--workload", choices=WORKLOADS, default="replica_sweep",
+                    help="another workload shape, timed alone on one GPU (default: the benchmarked sweep)")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.workload != "replica_sweep":
+        if world > 1:
+            raise SystemExit("--workload other than replica_sweep runs on one GPU")
+        return run_workload(args)
     if world > 1:
         import torch
         torch.cuda.set_device(local_rank)

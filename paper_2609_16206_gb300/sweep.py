@@ -143,3 +143,45 @@ def noise_sweep(wl, sigmas=NOISE_SIGMAS, seeds: int = 16, const_sets=None, polic
         ctr.ctr_gen_trace(wl.trace.replace(noise_sigma=float(sg)), seeds, 0, wl.n_req, view)
     run_step(None, wl.sim, const_sets, policies, R, wl.n_req, 0, buf, gen=False)
     return buf, R
+
+
+def calibration_sweep(sat_rates, widths=(3, 4, 5, 6, 7), mixes=(1.0, 5 / 6, 2 / 3, 1 / 2),
+                      loads=(0.8, 29 / 30, 17 / 15, 1.3), seeds: int = 16, n_req: int = 10_000,
+                      const_sets=None, device="cuda"):
+    """The mispriced-constants x pool-width sweep (sec. V-B, the calibration
+    study), batched: per pool width one trace buffer holds every (mix, load,
+    seed) replica -- replica (i * len(loads) + j) * seeds + s has mix i, load
+    j and sub-stream s -- and two simulation calls cover it: the learned
+    router under every constant set, and the three baselines under the
+    calibrated set.  `sat_rates[w][i]` is the saturation rate (milli-requests
+    per second) of width w and mix i; the offered rate is load x that.
+    Returns {width: (learned SweepBuffers, baseline SweepBuffers)}."""
+    const_sets = const_sets or W.mispriced_sets()
+    base_pols = [W.POLICY_RR, W.POLICY_JSQ, W.POLICY_HEURISTIC]
+    out = {}
+    for w in widths:
+        sc = W.SimCfg(n_prefill=2, n_decode=w)
+        R = len(mixes) * len(loads) * seeds
+        learned = alloc(sc, R, R * len(const_sets), n_req, device)
+        base = alloc(sc, R, R * len(base_pols), n_req, device)
+        for i, mix in enumerate(mixes):
+            for j, load in enumerate(loads):
+                rate = load_rate(sat_rates[w][i], load)
+                tc = W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(mix), rate_mreq=(rate, rate))
+                lo = (i * len(loads) + j) * seeds
+                view = {name: t[lo:lo + seeds] for name, t in learned.trace.items()}
+                ctr.ctr_gen_trace(tc, seeds, 0, n_req, view)
+        base.trace = learned.trace
+        run_step(None, sc, const_sets, [W.POLICY_LEARNED], R, n_req, 0, learned, gen=False)
+        run_step(None, sc, [W.CALIBRATED], base_pols, R, n_req, 0, base, gen=False)
+        learned.workspace = base.workspace = None  # released once the launches complete
+        out[w] = (learned, base)
+    return out
+
+
+def calibration_saturation(widths=(3, 4, 5, 6, 7), mixes=(1.0, 5 / 6, 2 / 3, 1 / 2), n_req: int = 10_000,
+                           device="cuda") -> dict:
+    """Saturation rate per (width, mix) for `calibration_sweep`."""
+    laws = [W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(m)) for m in mixes]
+    return {w: saturation_rate(laws, W.SimCfg(n_prefill=2, n_decode=w), n_req=n_req, device=device)
+            for w in widths}

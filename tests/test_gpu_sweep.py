@@ -147,3 +147,38 @@ def test_noise_sweep(orc):
     rr = [int(h[(i * seeds) * n_pol + 1]) for i in range(len(sweep.NOISE_SIGMAS))]
     lr = [int(h[(i * seeds) * n_pol + 0]) for i in range(len(sweep.NOISE_SIGMAS))]
     assert len(set(rr)) == 1 and len(set(lr)) == len(lr)
+
+
+def test_calibration_sweep_batched(orc):
+    """The batched calibration sweep: one trace buffer and two launches per width; sampled rows = oracle."""
+    ctr = need_gpu()
+    from paper_2609_16206_gb300 import sweep
+    widths, mixes, loads, seeds, n = (3, 6), (1.0, 0.5), (0.8, 1.3), 2, 1500
+    sat = sweep.calibration_saturation(widths, mixes, n_req=n)
+    out = sweep.calibration_sweep(sat, widths, mixes, loads, seeds, n_req=n)
+    torch.cuda.synchronize()
+    sets = W.mispriced_sets()
+    for w, (lb, bb) in out.items():
+        sc = W.SimCfg(n_prefill=2, n_decode=w)
+        st_l = lb.row_status.cpu().numpy()
+        h_l = lb.row_hash.cpu().numpy().astype(np.uint64)
+        st_b = bb.row_status.cpu().numpy()
+        h_b = bb.row_hash.cpu().numpy().astype(np.uint64)
+        for i, mix in enumerate(mixes):
+            for j, load in enumerate(loads):
+                r = (i * len(loads) + j) * seeds + (i + j) % seeds
+                trh = host_trace(lb.trace, r)
+                rate = sweep.load_rate(sat[w][i], load)
+                ref = orc.gen_trace(W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(mix), rate_mreq=(rate, rate)),
+                                    n, replica=(i + j) % seeds)
+                assert np.array_equal(trh["arrival_us"], ref["arrival_us"])
+                for si in (0, 21, 64):
+                    o = orc.simulate(sc, sets[si], W.POLICY_LEARNED, trh)
+                    assert st_l[r * len(sets) + si] == o["status"]
+                    if o["status"] == 0:
+                        assert int(h_l[r * len(sets) + si]) == o["hash"]
+                for b, pol in enumerate((W.POLICY_RR, W.POLICY_JSQ, W.POLICY_HEURISTIC)):
+                    o = orc.simulate(sc, W.CALIBRATED, pol, trh)
+                    assert st_b[r * 3 + b] == o["status"]
+                    if o["status"] == 0:
+                        assert int(h_b[r * 3 + b]) == o["hash"]
