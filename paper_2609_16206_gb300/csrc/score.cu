@@ -253,6 +253,29 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     const int tid = threadIdx.x;
     const int n_inst = P.n_inst;
 
+    // ---- stage the instance state first: it heads the critical path (state -> envelopes -> scoring), so
+    // its TMA bulk copy is issued before the request prefetch (plain loads when unaligned)
+    const uint32_t bytes = (uint32_t)n_inst * 4u;
+    const bool bulk = kVec && (bytes % 16u == 0) && (((uintptr_t)P.Q | (uintptr_t)P.A | (uintptr_t)P.kap) % 16u == 0);
+    const uint32_t bar = smem_addr(&sm.bar);
+    if (bulk && tid == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(3u * bytes) : "memory");
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                         smem_addr(sm.q)),
+                     "l"(P.Q), "r"(bytes), "r"(bar)
+                     : "memory");
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                         smem_addr(sm.a)),
+                     "l"(P.A), "r"(bytes), "r"(bar)
+                     : "memory");
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                         smem_addr(sm.kap)),
+                     "l"(P.kap), "r"(bytes), "r"(bar)
+                     : "memory");
+    }
+
     // the first two request vectors of this thread, in flight while the block builds its envelopes
     const int64_t nv = kVec ? (P.n >> 2) : 0;
     const int64_t stride = (int64_t)gridDim.x * kThreads;
@@ -275,32 +298,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         cn = ld_stream_u32(c4 + v + stride);
     }
 
-    // ---- stage the instance state: TMA bulk copy when aligned, else plain loads
-    const uint32_t bytes = (uint32_t)n_inst * 4u;
-    const bool bulk = kVec && (bytes % 16u == 0) && (((uintptr_t)P.Q | (uintptr_t)P.A | (uintptr_t)P.kap) % 16u == 0);
     if (bulk) {
-        const uint32_t bar = smem_addr(&sm.bar);
-        if (tid == 0) {
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        }
-        __syncthreads();
-        if (tid == 0) {
-            asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(3u * bytes)
-                         : "memory");
-            asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                             smem_addr(sm.q)),
-                         "l"(P.Q), "r"(bytes), "r"(bar)
-                         : "memory");
-            asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                             smem_addr(sm.a)),
-                         "l"(P.A), "r"(bytes), "r"(bar)
-                         : "memory");
-            asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                             smem_addr(sm.kap)),
-                         "l"(P.kap), "r"(bytes), "r"(bar)
-                         : "memory");
-        }
+        __syncthreads();  // the barrier is initialised before any thread polls it
         uint32_t done = 0;
         for (unsigned it = 0; it < kWaitLimit && !done; ++it) {
             asm volatile(
