@@ -30,9 +30,9 @@ REQUEST_FIELDS = (("arrival_us", torch.int64), ("prompt_len", torch.int32), ("tr
 
 
 class CtrError(RuntimeError):
-    def __init__(self, func, code):
+    def __init__(self, func, code, detail=None):
         self.code = code
-        super().__init__(f"{func} failed: {code} ({ctr_strerror(code)})")
+        super().__init__(f"{func} failed: {code} ({detail if detail is not None else ctr_strerror(code)})")
 
 
 # ---------------------------------------------------------------- C structs (ctr.h)
@@ -70,7 +70,7 @@ class CtrCostConsts(C.Structure):
                 ("backlog_signal", C.c_uint32), ("occupancy_poll_us", C.c_int64)]
 
 
-_lock = threading.Lock()
+_lock = threading.RLock()
 _lib = None
 
 
@@ -80,8 +80,8 @@ def lib():
     with _lock:
         if _lib is None:
             if not os.path.exists(LIB_PATH):
-                raise CtrError("load", CTR_ECUDA) from FileNotFoundError(
-                    f"{LIB_PATH} is missing: build it with paper_2609_16206_gb300/build.py")
+                msg = f"{LIB_PATH} is missing: build it with paper_2609_16206_gb300/build.py"
+                raise CtrError("load", CTR_ECUDA, detail=msg) from FileNotFoundError(msg)
             L = C.CDLL(LIB_PATH)
             vp, i32, i64 = C.c_void_p, C.c_int32, C.c_int64
             L.ctr_gen_trace.argtypes = [C.POINTER(CtrTraceCfg), i32, i64, i64, CtrRequests, vp]
@@ -106,9 +106,11 @@ def lib():
 
 
 def ctr_strerror(code: int) -> str:
+    if _lib is None and not os.path.exists(LIB_PATH):
+        return "libctr.so not loaded"
     try:
         return lib().ctr_strerror(int(code)).decode()
-    except CtrError:
+    except (CtrError, OSError):
         return "libctr.so not loaded"
 
 

@@ -79,3 +79,27 @@ def test_workspace_query_without_gpu_is_zero():
     from paper_2609_16206_gb300 import ctr
     from paper_2609_16206_gb300 import workloads as W
     assert ctr.ctr_workspace_bytes(0, W.SimCfg(), 4, 100) == 0
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """Without a built libctr.so the first call raises at once (it must not
+    fall back, and must not block on the loader's own lock)."""
+    import threading
+
+    from paper_2609_16206_gb300 import ctr
+    monkeypatch.setattr(ctr, "LIB_PATH", str(tmp_path / "libctr.so"))
+    monkeypatch.setattr(ctr, "_lib", None)
+    out = {}
+
+    def call():
+        try:
+            ctr.lib()
+        except ctr.CtrError as e:
+            out["err"] = e
+
+    t = threading.Thread(target=call, daemon=True)
+    t.start()
+    t.join(timeout=20)
+    assert not t.is_alive(), "loading a missing library blocked"
+    assert "err" in out and "is missing" in str(out["err"])
+    assert ctr.ctr_strerror(ctr.CTR_EINVAL) == "libctr.so not loaded"
