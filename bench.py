@@ -432,7 +432,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "d3d7298c094004a9": {"warp_inst": 165467741269, "dram_bytes": 32.14e9 + 21.94e9},
+    "616522b7e44dda88": {"warp_inst": 165095121660, "dram_bytes": 30.60e9 + 20.47e9},
 }
 
 

@@ -164,7 +164,8 @@ __device__ __forceinline__ int warp_argmin(uint64_t v)
 }
 
 struct Decode {
-    int64_t step_end, step_idx, kv_res, kv_rsv, R, ohat;
+    int64_t step_end, step_idx, R, ohat;
+    int32_t kv_res, kv_rsv;  // resident <= reserved <= C < 2^31 tokens
     uint64_t pend_top, act_top;
     int32_t n_act, q, pend_n, act_n, w_head, w_n;
     bool stepping;
@@ -222,7 +223,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 m = n <= kRecipN ? (int64_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n])) : room / n;
             }
             s.step_idx += m;
-            s.kv_res += m * n;
+            s.kv_res += (int32_t)(m * n);  // stays within the reservation
             s.R -= m * n;
             if (s.step_idx + 1 > P.max_steps) return CTR_ETIMEOUT;
             s.step_end += m * S;
@@ -246,8 +247,8 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 const int64_t ohk = __ldg(&P.trace.pred_out[tb + k]);
                 s.n_act -= 1;
                 s.q -= 1;
-                s.kv_res -= pk + ok;
-                s.kv_rsv -= pk + ok;
+                s.kv_res -= (int32_t)(pk + ok);
+                s.kv_rsv -= (int32_t)(pk + ok);
                 s.ohat -= ohk;
                 P.t_done[ob + k] = tev;
             }
@@ -267,8 +268,8 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 if (s.act_n == P.cap_act) return CTR_EOVERFLOW;
                 s.w_head = s.w_head + 1 == P.cap_wait ? 0 : s.w_head + 1;
                 s.w_n -= 1;
-                s.kv_rsv += pk + ok;
-                s.kv_res += pk;
+                s.kv_rsv += (int32_t)(pk + ok);
+                s.kv_res += (int32_t)pk;
                 s.n_act += 1;
                 heap_push(act, s.act_n, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
                 admitted += 1;
