@@ -6,7 +6,10 @@
 // met count and the TTFT range; the P99 is then selected exactly by a radix
 // select over (TTFT - min) with 11-bit digits, most significant first, each
 // pass histogramming the candidates that still match the digits chosen so far
-// (2048 shared-memory bins).  Rows are re-read from L2 by each pass.
+// (2048 shared-memory bins).  When the row fits (kStage), pass 0 also keeps
+// its TTFTs in shared memory as 32-bit values and the select passes read them
+// there, so a row crosses HBM once; a row with a TTFT outside [0, 2^32) or too
+// many requests re-reads its TTFTs from global memory instead.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -36,11 +39,13 @@ __device__ T block_reduce(T v, T identity, Op op, T* scratch)
     return r;
 }
 
+template <bool kStage>
 __global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P)
 {
     __shared__ uint32_t hist[kBins];
     __shared__ int64_t red64[kThreads / 32];
     __shared__ uint32_t pick[2];
+    extern __shared__ uint32_t ttft_s[];  // kStage: the row's TTFTs
     const int tid = threadIdx.x;
     const int64_t n = P.n_req;
 
@@ -48,17 +53,37 @@ __global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P
         const int64_t tb = (row / P.rows_per_replica) * n;
         const int64_t ob = row * n;
         int64_t met = 0, mn = INT64_MAX, mx = INT64_MIN;
-        for (int64_t k = tid; k < n; k += kThreads) {
-            const int64_t tf = P.t_first[ob + k];
-            const int64_t td = P.t_done[ob + k];
-            const int64_t ttft = tf - P.trace.arrival_us[tb + k];
-            const int64_t o = P.trace.true_out[tb + k];
-            int c = P.trace.slo_class[tb + k];
-            if (c >= P.n_classes) c = P.n_classes - 1;
-            const bool ok = ttft <= P.ttft[c] && (o == 1 || td - tf <= P.tpot[c] * (o - 1));
-            met += ok;
-            mn = ttft < mn ? ttft : mn;
-            mx = ttft > mx ? ttft : mx;
+        // 4 elements per thread per round, all loads issued before any is used (the pass is latency-bound)
+        for (int64_t base = tid; base < n; base += (int64_t)kThreads * 4) {
+            int64_t tf[4], td[4], ta[4];
+            int32_t ov[4];
+            uint32_t cv[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t k = base + (int64_t)u * kThreads;
+                if (k < n) {
+                    tf[u] = __ldg(&P.t_first[ob + k]);
+                    td[u] = __ldg(&P.t_done[ob + k]);
+                    ta[u] = __ldg(&P.trace.arrival_us[tb + k]);
+                    ov[u] = __ldg(&P.trace.true_out[tb + k]);
+                    cv[u] = __ldg(&P.trace.slo_class[tb + k]);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t k = base + (int64_t)u * kThreads;
+                if (k < n) {
+                    const int64_t ttft = tf[u] - ta[u];
+                    const int64_t o = ov[u];
+                    int c = (int)cv[u];
+                    if (c >= P.n_classes) c = P.n_classes - 1;
+                    const bool ok = ttft <= P.ttft[c] && (o == 1 || td[u] - tf[u] <= P.tpot[c] * (o - 1));
+                    met += ok;
+                    mn = ttft < mn ? ttft : mn;
+                    mx = ttft > mx ? ttft : mx;
+                    if (kStage) ttft_s[k] = (uint32_t)ttft;
+                }
+            }
         }
         met = block_reduce<int64_t>(met, 0, [](int64_t a, int64_t b) { return a + b; }, red64);
         mn = block_reduce<int64_t>(mn, INT64_MAX, [](int64_t a, int64_t b) { return a < b ? a : b; }, red64);
@@ -70,6 +95,8 @@ __global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P
             }
             continue;
         }
+        // the staged 32-bit copies are exact when every TTFT lies in [0, 2^32)
+        const bool staged = kStage && mn >= 0 && mx < (int64_t(1) << 32);
         const uint64_t range = (uint64_t)mx - (uint64_t)mn;
         int shift = range == 0 ? 0 : 64 - __clzll((long long)range);  // bits still undetermined
         uint64_t prefix = 0;                                            // chosen high bits of (ttft - mn)
@@ -82,7 +109,8 @@ __global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P
             __syncthreads();
             const uint32_t dmask = (1u << dbits) - 1u;
             for (int64_t k = tid; k < n; k += kThreads) {
-                const uint64_t v = (uint64_t)(P.t_first[ob + k] - P.trace.arrival_us[tb + k]) - (uint64_t)mn;
+                const uint64_t v = (staged ? (uint64_t)ttft_s[k] : (uint64_t)(P.t_first[ob + k] - P.trace.arrival_us[tb + k])) -
+                                   (uint64_t)mn;
                 const bool match = above >= 64 || (v >> above) == (prefix >> above);
                 if (match) atomicAdd(&hist[(uint32_t)(v >> shift) & dmask], 1u);
             }
@@ -139,9 +167,23 @@ cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream)
     if (err != cudaSuccess) return err;
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
+    constexpr int64_t kStageMaxBytes = 160 * 1024;  // a row's TTFTs staged in shared memory up to this
+    const int64_t stage_bytes = p.n_req * 4;
+    if (stage_bytes > 0 && stage_bytes <= kStageMaxBytes) {
+        err = cudaFuncSetAttribute(goodput_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)stage_bytes);
+        if (err != cudaSuccess) return err;
+        int per_sm = 0;
+        err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, goodput_kernel<true>, kThreads, (size_t)stage_bytes);
+        if (err != cudaSuccess) return err;
+        int64_t blocks = p.n_rows;
+        const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+        if (blocks > cap) blocks = cap;
+        goodput_kernel<true><<<(unsigned)blocks, kThreads, (size_t)stage_bytes, stream>>>(p);
+        return cudaGetLastError();
+    }
     int64_t blocks = p.n_rows;
     if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
-    goodput_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(p);
+    goodput_kernel<false><<<(unsigned)blocks, kThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
 
