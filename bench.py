@@ -148,12 +148,36 @@ def run_reference(args, rank, world):
 SIM_SOURCES = ("paper_2609_16206_gb300/csrc/sim.cu", "paper_2609_16206_gb300/csrc/ctr_internal.cuh", "include/ctr.h")
 
 
+def _strip_comments(src: str) -> str:
+    """C/C++ source without comments and trailing blanks (string and character
+    literals kept), so that editing a comment does not change the key."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    return "\n".join(line.rstrip() for line in "".join(out).splitlines() if line.strip())
+
+
 def _source_hash() -> str:
-    """Hash of the files that define the simulator kernel."""
+    """Hash of the code (comments stripped) of the files that define the simulator kernel."""
     h = hashlib.sha256()
     for rel in SIM_SOURCES:
-        with open(os.path.join(ROOT, rel), "rb") as f:
-            h.update(rel.encode() + f.read())
+        with open(os.path.join(ROOT, rel), encoding="utf-8") as f:
+            h.update(rel.encode() + _strip_comments(f.read()).encode())
     return h.hexdigest()[:16]
 
 
@@ -432,7 +456,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "616522b7e44dda88": {"warp_inst": 165095121660, "dram_bytes": 30.60e9 + 20.47e9},
+    "f6e82b0057fb492f": {"warp_inst": 165095121660, "dram_bytes": 30.60e9 + 20.47e9},
 }
 
 

@@ -3,17 +3,21 @@
 // with the continuous decode batching of sec. VI, the marginal-cost score of
 // sec. III-A and the sec. IV-C baselines.
 //
-// Layout: one warp simulates one row (replica x cost-constant set x policy);
-// lane i < n_pre is prefill instance i, lane n_pre + d is decode instance d.
-// Warps are persistent and pull rows from an atomic counter in the workspace,
-// so rows of different length balance across the GPU.  For every arrival k:
+// Layout: a row is (replica x cost-constant set x policy); a lane group of G
+// lanes (G = the next power of two >= the pool size) simulates one row, lane
+// i < n_pre being prefill instance i and lane n_pre + d decode instance d, and
+// a warp carries 32 / G rows side by side (the policies of one replica, which
+// share arrival times).  Warps are persistent and pull row groups from an
+// atomic counter in the workspace.  For every arrival k:
 //   1. each decode lane advances its own instance's event loop to t_k
-//      (step ends, KV-ready events, FCFS admissions, step starts);
-//      each prefill lane retires prefills that ended by t_k;
-//   2. every lane prices its instance for the policy, and two warp-wide
-//      argmins (redux.sync, ties to the lowest lane) pick i_pre and i_dec;
-//   3. the i_pre lane commits the FCFS prefill, broadcasts the KV-ready time,
-//      and the i_dec lane queues the request.
+//      (runs of plain steps in closed form, step ends, KV-ready requests,
+//      FCFS admissions, step starts); each prefill lane retires prefills that
+//      ended by t_k (or, with batched prefill, ends and starts its batches
+//      first and hands the members' KV-ready times to the decode lanes);
+//   2. every lane prices its instance for the row's policy, and two argmins
+//      within the lane group (ties to the lowest lane) pick i_pre and i_dec;
+//   3. the i_pre lane commits the prefill, broadcasts the KV-ready time when
+//      it is known, and the i_dec lane queues the request.
 // All time and cost arithmetic is int64 fixed point, so every decision is
 // deterministic.  Instances never interact except through routing, so the
 // per-lane event loops reproduce the global event order exactly (events at
@@ -23,10 +27,12 @@
 // [entry][lane] so that the lanes' heap tops share cache lines: a min-heap of
 // pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
 // lanes use the same region as their in-flight ring of prefill end times,
-// packed with the prompt length as end << 21 | p),
-// a min-heap of active requests keyed by finishing step (finish << 23 | k),
-// and a FIFO ring of KV-ready requests awaiting admission.  Heap tops are
-// cached in registers, so a plain decode step touches no memory.
+// packed with the prompt length as end << 21 | p), a min-heap of active
+// requests keyed by finishing step (finish << 23 | k), and a FIFO ring of
+// KV-ready requests awaiting admission.  Heap tops are cached in registers,
+// so a run of plain decode steps touches no memory.  The row checksum's
+// routing terms are summed here; its first-token and completion terms are
+// summed by hash_kernel from the outputs.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -195,11 +201,11 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                                               uint32_t* wait, int64_t tb, int64_t ob)
 {
     for (;;) {
-        // Plain step ends first, in a tight loop: the step ends by T, no request
-        // finishes with it, nothing becomes KV-ready at that instant and nobody
-        // waits for admission, so the batch is unchanged and the next step
-        // starts at once.  Lanes leave this loop at their next non-plain event;
-        // the general handler below then runs once for all of them together.
+        // Plain step ends first: the step ends by T, no request finishes with
+        // it, nothing has become KV-ready by then and nobody waits for
+        // admission, so the batch is unchanged and the next step starts at
+        // once.  Lanes leave this loop at their next non-plain event, which
+        // the handler below takes.
         const int64_t tp = s.pend_n > 0 ? (int64_t)(s.pend_top >> kKeyBits) : kNever;
         const int64_t limit = tp <= T ? tp - 1 : T;  // plain step ends lie at or before limit
         // The run is taken in closed form: while the floor(KV / kv_div) term of
