@@ -19,7 +19,8 @@ def _goodput(ctr, sc, tr, R, rows_per, N, tf, td):
 
 
 @pytest.mark.parametrize("wl,R,N", [(W.single_replica(), 1, 2000), (W.replica_sweep(), 8, 5000),
-                                    (W.large_pool(rate_mreq=34_000), 2, 3000), (W.replica_sweep(), 3, 37)])
+                                    (W.large_pool(rate_mreq=34_000), 2, 3000), (W.replica_sweep(), 3, 37),
+                                    (W.replica_sweep(), 1, 45_000)])  # rows past the shared-memory staging
 def test_goodput_matches_oracle(orc, wl, R, N):
     ctr = need_gpu()
     tr = gen(ctr, wl.trace, R, N)
@@ -40,7 +41,7 @@ def test_goodput_adversarial_times(orc):
     ctr = need_gpu()
     rng = np.random.default_rng(8)
     sc = W.SimCfg(n_classes=3, ttft_slo_us=(10, 10**6, 10**12), tpot_slo_us=(0, 5, 10**9))
-    for N in (1, 2, 100, 101, 4097):
+    for N in (1, 2, 100, 101, 4097, 45_000):  # 45,000: rows too long to stage in shared memory
         R = 3
         trh = {"arrival_us": np.sort(rng.integers(0, 10**6, (R, N)), axis=1), "prompt_len": np.ones((R, N)),
                "true_out": rng.integers(1, 4, (R, N)), "pred_out": np.ones((R, N)),
