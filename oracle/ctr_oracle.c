@@ -561,7 +561,7 @@ static int64_t argmin_lowest(const int64_t* v, int64_t n)
 }
 
 /* B_d = floor(R_d * step_d / max(1, n_d)), saturated at 2^40 [reading: the
- * "true remaining work" of sec. VI priced at the current batch step time] */
+ * true remaining work of sec. VI, priced at the current batch step time] */
 static int64_t decode_backlog(int64_t remaining, int64_t step, int64_t n_active)
 {
     unsigned __int128 prod = (unsigned __int128)(uint64_t)remaining * (uint64_t)step;
@@ -602,7 +602,7 @@ static void p2_candidates(int64_t k, int64_t t, int64_t np, int64_t c[2])
     p2_pair(w[2], w[3], np, c);
 }
 
-/* Batched prefill (sec. VI: continuous batching "in both stages") [reading]:
+/* Batched prefill (sec. VI batches the prefill stage as well as the decode stage) [reading]:
  * an instance runs one batch at a time.  A batch takes, FCFS from the
  * instance's queue, the head request and then every next request while the
  * batch's prompt tokens stay within pre_batch_tokens; it lasts
@@ -664,9 +664,9 @@ static int64_t batched_backlog_pre(const sim_t* s, int64_t i, int64_t t)
     return b;
 }
 
-/* Backlog as the deployed proxy sees it [reading: sec. IV-A's in-flight
- * ledger "yielding seconds-of-backlog", priced with the router's own
- * constants as sec. VI describes]: the sum over requests routed to the
+/* Backlog as the deployed proxy sees it [reading: sec. IV-A's ledger of
+ * in-flight requests, from which the proxy derives seconds of backlog, priced
+ * with the router's own constants as sec. VI describes]: the sum over requests routed to the
  * instance and still in flight there of their priced work, each priced once
  * at admission and never decremented.  Prefill: tau_pre0 + tau_pre * p until
  * the prefill ends; decode: o_hat * tau_dec until the request completes (o_hat
