@@ -6,8 +6,8 @@
   path for a workload: trace generation, simulation under every policy and
   constant set, goodput.
 * ``saturation_rate`` -- the arrival rate at which round-robin goodput
-  crosses 1/2 (the paper drives every workload at the rate where round-robin
-  is "mid-collapse", found by probing, sec. IV-B): an integer bisection over
+  crosses 1/2 (sec. IV-B runs each workload at the load where round-robin is
+  half-way into collapse, located by probing): an integer bisection over
   milli-requests per second, every probe a GPU simulation.
 * ``calibration_sweep_cfgs`` / ``load_rate`` -- the mispriced-constants x
   pool-width sweep grid and its offered rates.
