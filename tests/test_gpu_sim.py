@@ -310,3 +310,38 @@ def test_workload_families_batched_prefill(orc, wl):
     sets = [wl.consts[0], W.as_deployed(wl.consts[0])]
     res = simulate(ctr, sc, sets, ALL_FIVE, tr, R, N)
     _check_rows(orc, sc, sets, ALL_FIVE, [host_trace(tr, r) for r in range(R)], res, N)
+
+
+def _full_size_sampled(orc, wl, sets, samples):
+    ctr = need_gpu()
+    R, N = wl.n_replicas, wl.n_req
+    pols = list(W.ALL_POLICIES)
+    tr = gen(ctr, wl.trace, R, N)
+    rows = R * len(sets) * len(pols)
+    tf = torch.empty((rows, N), dtype=torch.int64, device="cuda")
+    td = torch.empty_like(tf)
+    h = torch.empty(rows, dtype=torch.int64, device="cuda")
+    st = torch.empty(rows, dtype=torch.int32, device="cuda")
+    ws = ctr.simulate_workspace(wl.sim, rows, N, "cuda")
+    ctr.ctr_simulate(wl.sim, sets, pols, tr, R, N, tf, td, h, st, ws)
+    torch.cuda.synchronize()
+    assert int((st != 0).sum()) == 0
+    hh = h.cpu().numpy().astype(np.uint64)
+    for r in samples:
+        trh = host_trace(tr, r)
+        for si, cc in enumerate(sets):
+            for j, pol in enumerate(pols):
+                o = orc.simulate(wl.sim, cc, pol, trh)
+                assert o["status"] == 0 and int(hh[(r * len(sets) + si) * len(pols) + j]) == o["hash"], (r, si, pol)
+
+
+def test_full_size_document_batched_prefill_sampled(orc):
+    """4,096 document replicas x 10,000 requests with batched prefill, one launch of the
+    extended kernel; sampled rows against the oracle."""
+    _full_size_sampled(orc, W.document(n_replicas=4096), [W.CALIBRATED], (0, 1, 2047, 4095))
+
+
+def test_full_size_deployed_signals_sampled(orc):
+    """The benchmarked sweep under the deployed proxy's signals (ledger backlog, 50 ms
+    occupancy poll) beside the true ones, 4,096 x 20,000 in one launch; sampled rows."""
+    _full_size_sampled(orc, W.replica_sweep(), [W.CALIBRATED, W.as_deployed(W.CALIBRATED)], (0, 3, 4095))
