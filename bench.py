@@ -486,11 +486,12 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "f6e82b0057fb492f": {"warp_inst": 165095121660, "dram_bytes": 30.60e9 + 20.47e9},
+    "4fb6926186954286": {"warp_inst": 164340141282, "dram_bytes": 30.59e9 + 20.45e9},
 }
 
 
-WORKLOADS = ("replica_sweep", "single_replica", "large_pool", "calibration_sweep", "document")
+WORKLOADS = ("replica_sweep", "single_replica", "large_pool", "calibration_sweep", "document", "deployed_signals",
+             "power_of_two", "noise_sweep")
 
 
 def run_workload(args):
@@ -508,7 +509,18 @@ def run_workload(args):
     stream = torch.cuda.current_stream()
     name = args.workload
     info = {}
-    if name == "calibration_sweep":
+    if name == "noise_sweep":
+        base = W.replica_sweep(n_req=args.requests or 20_000)
+        seeds = args.replicas or 512
+        n_sig = len(sweep.NOISE_SIGMAS)
+        routed = n_sig * seeds * len(W.ALL_POLICIES) * base.n_req
+        cfg = {"workload": f"noise_sweep_2p6d_{n_sig}x{seeds}x{base.n_req}", "noise_sigmas": list(sweep.NOISE_SIGMAS),
+               "replicas": n_sig * seeds, "requests_per_replica": base.n_req, "policies": len(W.ALL_POLICIES)}
+        state = {}
+
+        def step():
+            state["out"] = sweep.noise_sweep(base, seeds=seeds)
+    elif name == "calibration_sweep":
         t_sat = time.perf_counter()
         sat = sweep.calibration_saturation()
         torch.cuda.synchronize()
@@ -527,6 +539,13 @@ def run_workload(args):
             wl = W.single_replica()
         elif name == "document":
             wl = W.document(n_replicas=args.replicas or 4096, n_req=args.requests or 10_000)
+        elif name in ("deployed_signals", "power_of_two"):
+            wl = W.replica_sweep(n_replicas=args.replicas or 4096, n_req=args.requests or 20_000)
+            if name == "deployed_signals":
+                wl = dataclasses.replace(wl, name=wl.name + "_deployed", consts=[W.as_deployed(W.CALIBRATED)])
+            else:
+                wl = dataclasses.replace(wl, name=wl.name + "_p2",
+                                         policies=(W.POLICY_LEARNED_P2, W.POLICY_RR, W.POLICY_JSQ, W.POLICY_HEURISTIC))
         elif name == "large_pool":
             base = W.large_pool(n_replicas=args.replicas or 16384, n_req=args.requests or 50_000)
             t_sat = time.perf_counter()
@@ -536,7 +555,7 @@ def run_workload(args):
             wl = dataclasses.replace(base, trace=base.trace.replace(rate_mreq=(info["rate_mreq"],) * 2))
         else:
             wl = W.replica_sweep(n_replicas=args.replicas or 4096, n_req=args.requests or 20_000)
-        pols = list(W.ALL_POLICIES)
+        pols = list(wl.policies)
         rows = wl.n_replicas * len(wl.consts) * len(pols)
         routed = rows * wl.n_req
         buf = sweep.alloc(wl.sim, wl.n_replicas, rows, wl.n_req, dev)
@@ -562,6 +581,8 @@ def run_workload(args):
     ms_step = t0.elapsed_time(t1) / args.steps
     if name == "calibration_sweep":
         failed = sum(int((b.row_status != 0).sum()) for pair in state["out"].values() for b in pair)
+    elif name == "noise_sweep":
+        failed = int((state["out"][0].row_status != 0).sum())
     else:
         failed = int((buf.row_status != 0).sum())
     cfg.update(info)

@@ -196,9 +196,12 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
 // Advance one decode instance through every event at times <= T.  The pending
 // heap may hold requests already KV-ready (taken at the next step end); it has
 // room for cap_pend + cap_wait + 1 entries, so a full heap means the waiting
-// FIFO has overflowed.
+// FIFO has overflowed.  kSnap: when tsnap >= 0, also record in kv_snap the
+// resident KV as it is after every event at times <= tsnap (an occupancy
+// poll; tsnap <= T), then set tsnap to -1.
+template <bool kSnap>
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
-                                              uint32_t* wait, int64_t tb, int64_t ob)
+                                              uint32_t* wait, int64_t tb, int64_t ob, int64_t& tsnap, int64_t& kv_snap)
 {
     for (;;) {
         // Plain step ends first: the step ends by T, no request finishes with
@@ -228,6 +231,21 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             if (m * n > room) {  // the KV term changes first: m = floor(room / n) >= 1
                 m = n <= kRecipN ? (int64_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n])) : room / n;
             }
+            if constexpr (kSnap) {
+                // the poll instant falls before this run or inside it: the occupancy
+                // there follows from the number of the run's ends by then
+                if (tsnap >= 0) {
+                    if (tsnap < s.step_end) {
+                        kv_snap = s.kv_res;
+                        tsnap = -1;
+                    } else if (tsnap < s.step_end + (m - 1) * S) {
+                        const int64_t d = tsnap - s.step_end;  // < (m - 1) S < 2^57
+                        const int64_t j = (d < (int64_t(1) << 56) ? floor_div_small(d, S) : d / S) + 1;
+                        kv_snap = s.kv_res + j * n;
+                        tsnap = -1;
+                    }
+                }
+            }
             s.step_idx += m;
             s.kv_res += (int32_t)(m * n);  // stays within the reservation
             s.R -= m * n;
@@ -239,6 +257,12 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
         // next admission), so it is taken there, in the same pass: the next
         // event is the running step's end, or the next KV-ready when idle.
         const int64_t tev = s.stepping ? s.step_end : tp;
+        if constexpr (kSnap) {
+            if (tsnap >= 0 && tev > tsnap) {  // every event by the poll instant is done
+                kv_snap = s.kv_res;
+                tsnap = -1;
+            }
+        }
         if (tev > T) return CTR_OK;
         if (s.stepping) {  // (1) the running step ends: one token for every active request
             s.step_idx += 1;
@@ -518,18 +542,18 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 }
                 if (live) {
                     if (is_dec) {
+                        int64_t tsnap = -1;
                         if (kExt && cc.poll_us > 0) {
                             // the router sees the occupancy of the last poll instant floor(T / D) D,
-                            // taken after every event at that instant: advance there first
+                            // taken after every event at that instant, on the way to T
                             const int64_t tp = (int64_t)div_recip((uint64_t)T, (uint64_t)cc.poll_us, cc.poll_recip) *
                                                cc.poll_us;
-                            if (err == CTR_OK && tp > last_poll) {
-                                err = decode_advance(s, tp, P, pend, act, wait, tb, ob);
-                                kv_seen = s.kv_res;
+                            if (tp > last_poll) {
+                                tsnap = tp;
                                 last_poll = tp;
                             }
                         }
-                        if (err == CTR_OK) err = decode_advance(s, T, P, pend, act, wait, tb, ob);
+                        if (err == CTR_OK) err = decode_advance<kExt>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen);
                     } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
                         while (ring_n > 0 && ring_front <= thr) {
@@ -711,7 +735,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
             }
         }
-        if (live && is_dec) err = decode_advance(s, kNever - 1, P, pend, act, wait, tb, ob);
+        if (live && is_dec) {
+            int64_t no_snap = -1;
+            err = decode_advance<false>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen);
+        }
 
 #pragma unroll
         for (int off = G / 2; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off, G);
