@@ -41,7 +41,8 @@ def _check(orc, p, oh, cls, Q, A, kap, consts, am, cost):
     bad_cls = cls >= 4
     assert np.all(am[bad_cls] == -1) and np.all(np.isnan(cost[bad_cls]))
     ok = ~bad_cls
-    gap = (second - best) / best
+    with np.errstate(divide="ignore", invalid="ignore"):  # a zero minimum: inf (strict) or nan (a tie)
+        gap = (second - best) / best
     strict = ok & (gap >= REL_GAP)
     assert np.array_equal(am[strict], ref_am[strict]), np.flatnonzero(am[strict] != ref_am[strict])[:5]
     idx = np.flatnonzero(ok)
@@ -131,3 +132,31 @@ def test_invalid_arguments():
     big = torch.zeros(257, device="cuda")
     with pytest.raises(ctr.CtrError):
         ctr.ctr_score_batch(x, x, c, big, big, big, W.SCORE_CONSTS, am, x)
+
+
+@pytest.mark.parametrize("seed", range(48))
+def test_random_scoring_problems(orc, seed):
+    """Seeded random problems: 1-256 instances (duplicated ones give exact ties), constants with zero
+    weights, classes including invalid ones, aligned and misaligned buffers."""
+    ctr = need_gpu()
+    rng = np.random.default_rng(500 + seed)
+    n_inst = int(rng.choice([1, 2, 5, 17, 64, 65, 130, 256]))
+    n = int(rng.choice([0, 1, 7, 1000, 20_001]))
+    p = np.floor(rng.exponential(800.0, n)).astype(np.float32)
+    oh = np.floor(rng.exponential(400.0, n) + rng.integers(0, 2, n)).astype(np.float32)
+    cls = rng.integers(0, 5 if seed % 3 == 0 else 4, n).astype(np.uint8)
+    Q = rng.integers(0, 1 << int(rng.integers(1, 17)), n_inst).astype(np.float32)
+    A = rng.integers(0, 1 << int(rng.integers(1, 9)), n_inst).astype(np.float32)
+    kap = rng.random(n_inst, dtype=np.float32)
+    if n_inst > 1 and seed % 4 == 1:  # duplicated instances: exact ties broken by index
+        j = rng.integers(0, n_inst, n_inst // 2)
+        Q[j], A[j], kap[j] = Q[0], A[0], kap[0]
+    consts = W.SCORE_CONSTS.copy()
+    consts[:9] *= rng.choice([0.0, 0.5, 1.0, 3.0], 9).astype(np.float32)
+    consts[8] = np.float32(1.0 / float(rng.choice([1e4, 2e5, 1e6])))
+    consts[9:] = rng.choice([0.5, 1.0, 2.0], 4).astype(np.float32)
+    if consts[:8].max() == 0:
+        consts[0] = 1.0
+    am, cost = _run(ctr, p, oh, cls, Q, A, kap, consts, offset=int(seed % 2))
+    if n:
+        _check(orc, p, oh, cls, Q, A, kap, consts, am, cost)
