@@ -5,6 +5,7 @@ GPU and by the oracle, compared row by row (status, checksum, and every time
 and route)."""
 import numpy as np
 import pytest
+import torch
 
 from gpuutil import gen, host_trace, need_gpu, simulate
 from paper_2609_16206_gb300 import workloads as W
@@ -56,6 +57,12 @@ def test_random_configuration(orc, seed):
     sc, tc, sets, pols, R, N = _case(rng)
     tr = gen(ctr, tc, R, N)
     res = simulate(ctr, sc, sets, pols, tr, R, N)
+    rows = R * len(sets) * len(pols)
+    met = torch.empty(rows, dtype=torch.int64, device="cuda")
+    p99 = torch.empty(rows, dtype=torch.int64, device="cuda")
+    ctr.ctr_goodput(sc, tr, R, len(sets) * len(pols), N, torch.from_numpy(res["t_first_us"]).cuda(),
+                    torch.from_numpy(res["t_done_us"]).cuda(), met, p99)
+    met, p99 = met.cpu().numpy(), p99.cpu().numpy()
     row = 0
     for r in range(R):
         trh = host_trace(tr, r)
@@ -70,4 +77,5 @@ def test_random_configuration(orc, seed):
                     assert int(res["hash"][row]) == o["hash"], (seed, row)
                     for key in ("t_first_us", "t_done_us", "i_pre", "i_dec"):
                         assert np.array_equal(res[key][row], o[key]), (seed, row, key)
+                    assert (met[row], p99[row]) == orc.goodput(sc, trh, o["t_first_us"], o["t_done_us"]), (seed, row)
                 row += 1
