@@ -486,7 +486,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "4fb6926186954286": {"warp_inst": 164340141282, "dram_bytes": 30.59e9 + 20.45e9},
+    "ba5dc650cdbd67a7": {"warp_inst": 164340141282, "dram_bytes": 30.62e9 + 20.48e9},
 }
 
 

@@ -375,9 +375,9 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // workload have the same number of requests, so the groups walk their
 // arrivals in lockstep (request k of every row at once, each at its own time);
 // the per-lane event loops, the per-group argmins and the commits are
-// independent across groups.  kExt compiles in the deployed proxy's
-// signals (ledger backlog, polled occupancy) and batched prefill; the host
-// launches that instantiation only when a launch asks for one of them.
+// independent across groups.  kMode 1 compiles in the deployed proxy's
+// signals (ledger backlog, polled occupancy), kMode 2 batched prefill as
+// well; the host launches the least instantiation a launch needs.
 //
 // Batched prefill: a prefill lane's ring holds its in-flight requests as
 // k << 26 | d << 21 | p (running batch first, then the queue).  Before the
@@ -386,9 +386,11 @@ __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 // (contiguous at the ring's head) is published to the group, and every
 // decode lane copies its own members, now with known KV-ready times, into its
 // pending heap.  Repeated until no prefill lane has another batch ending.
-template <int G, bool kExt, int kBlocksPerSM>
+template <int G, int kMode, int kBlocksPerSM>
 __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(const __grid_constant__ SimParams P)
 {
+    constexpr bool kSig = kMode >= 1;  // the proxy's signals: ledger backlog, polled occupancy
+    constexpr bool kBat = kMode == 2;  // batched prefill
     constexpr int kRowsPerWarp = 32 / G;
     const int lane = threadIdx.x & 31;
     const int grp = lane / G;
@@ -447,7 +449,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         // queue behind it, cut FCFS into budget-limited batches, forms q_batches, the last of q_tail tokens
         int32_t run_n = 0, q_batches = 0;
         int64_t run_p = 0, q_tail = 0;
-        const bool batched = kExt && P.pre_batch > 0;
+        const bool batched = kBat && P.pre_batch > 0;
 
         // Batched prefill: end every batch that ends by T, start the next at that
         // instant, and hand the members' KV-ready times to their decode lanes
@@ -537,13 +539,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 const int64_t ohk = __shfl_sync(kFull, my_oh, j, G);
 
                 // 1. advance every instance to the arrival time
-                if constexpr (kExt) {
+                if constexpr (kBat) {
                     if (batched) prefill_batches(T);
                 }
                 if (live) {
                     if (is_dec) {
                         int64_t tsnap = -1;
-                        if (kExt && cc.poll_us > 0) {
+                        if (kSig && cc.poll_us > 0) {
                             // the router sees the occupancy of the last poll instant floor(T / D) D,
                             // taken after every event at that instant, on the way to T
                             const int64_t tp = (int64_t)div_recip((uint64_t)T, (uint64_t)cc.poll_us, cc.poll_recip) *
@@ -553,11 +555,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 last_poll = tp;
                             }
                         }
-                        if (err == CTR_OK) err = decode_advance<kExt>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen);
+                        if (err == CTR_OK) err = decode_advance<kSig>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen);
                     } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
                         while (ring_n > 0 && ring_front <= thr) {
-                            if constexpr (kExt) ring_sum_p -= ring_front & kRingPMask;
+                            if constexpr (kSig) ring_sum_p -= ring_front & kRingPMask;
                             ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
                             ring_n -= 1;
                             ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
@@ -583,7 +585,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                     P.pre_tok * (ring_sum_p - run_p);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            if (kExt && cc.proxy) {  // the ledger: tau_pre0 + tau_pre p per prefill not yet ended
+                            if (kSig && cc.proxy) {  // the ledger: tau_pre0 + tau_pre p per prefill not yet ended
                                 b = cc.tau_pre0 * (int64_t)ring_n + cc.tau_pre * ring_sum_p;
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
@@ -607,11 +609,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                                                       : lo / nd);
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            if (kExt && cc.proxy) {  // the ledger: tau_dec o_hat per request routed here and not done
+                            if (kSig && cc.proxy) {  // the ledger: tau_dec o_hat per request routed here and not done
                                 b = (cc.ablate & CTR_ABLATE_PREDICTED_LENGTH) ? 0 : cc.tau_dec * s.ohat;
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
-                            const int64_t kv = kExt && cc.poll_us > 0 ? kv_seen : s.kv_res;
+                            const int64_t kv = kSig && cc.poll_us > 0 ? kv_seen : s.kv_res;
                             int64_t press = (int64_t)div_recip((uint64_t)(kv + pk + oh_f) << 16,
                                                                (uint64_t)P.kv_cap, P.kv_cap_recip);
                             if (press > kPressureClamp) press = kPressureClamp;
@@ -699,7 +701,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         ring[pos * kWarp] = e;
                         if (ring_n == 0) ring_front = e;
                         ring_n += 1;
-                        if constexpr (kExt) ring_sum_p += pk;
+                        if constexpr (kSig) ring_sum_p += pk;
                     }
                 }
                 ready = __shfl_sync(kFull, ready, ip, G);
@@ -729,7 +731,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
             }
         }
         // drain: every remaining batch, then every remaining event
-        if constexpr (kExt) {
+        if constexpr (kBat) {
             if (batched) {
                 prefill_batches(kNever - 1);
                 if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
@@ -808,13 +810,14 @@ int sim_max_resident_warps(int* warps_per_block, int* blocks)
     int dev = 0, sms = 0, per_sm = 0, per_sm_g = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    // the smallest occupancy over the group widths at 8 blocks per SM, so one
-    // workspace size fits every launch
+    // the smallest occupancy over the group widths and modes at 8 blocks per
+    // SM, so one workspace size fits every launch
     per_sm = 1 << 30;
-    const void* kernels[8] = {(const void*)sim_kernel<4, false, 8>, (const void*)sim_kernel<8, false, 8>,
-                              (const void*)sim_kernel<16, false, 8>, (const void*)sim_kernel<32, false, 8>,
-                              (const void*)sim_kernel<4, true, 8>, (const void*)sim_kernel<8, true, 8>,
-                              (const void*)sim_kernel<16, true, 8>, (const void*)sim_kernel<32, true, 8>};
+    const void* kernels[12] = {
+        (const void*)sim_kernel<4, 0, 8>, (const void*)sim_kernel<8, 0, 8>, (const void*)sim_kernel<16, 0, 8>,
+        (const void*)sim_kernel<32, 0, 8>, (const void*)sim_kernel<4, 1, 8>, (const void*)sim_kernel<8, 1, 8>,
+        (const void*)sim_kernel<16, 1, 8>, (const void*)sim_kernel<32, 1, 8>, (const void*)sim_kernel<4, 2, 8>,
+        (const void*)sim_kernel<8, 2, 8>, (const void*)sim_kernel<16, 2, 8>, (const void*)sim_kernel<32, 2, 8>};
     for (const void* k : kernels) {
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_g, k, kWarpsPerBlock * 32, 0) != cudaSuccess)
             return 0;
@@ -830,20 +833,31 @@ namespace {
 // 7 blocks per SM (72 registers a thread, fewer spills) when all of the
 // launch's persistent warps fit on the GPU at that occupancy -- the common
 // case of one row group per warp -- else 8 (more warps to hide latency).
-template <int G, bool kExt>
+template <int G, int kMode>
 cudaError_t launch_width(const SimParams& p, int blocks, cudaStream_t stream)
 {
     int dev = 0, sms = 0, per_sm7 = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return cudaErrorInvalidDevice;
     cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm7, sim_kernel<G, kExt, 7>, kWarpsPerBlock * 32, 0);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm7, sim_kernel<G, kMode, 7>, kWarpsPerBlock * 32, 0);
     if (e != cudaSuccess) return e;
     if ((int64_t)p.n_slots <= (int64_t)sms * per_sm7 * kWarpsPerBlock)
-        sim_kernel<G, kExt, 7><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
+        sim_kernel<G, kMode, 7><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
     else
-        sim_kernel<G, kExt, 8><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
+        sim_kernel<G, kMode, 8><<<blocks, kWarpsPerBlock * 32, 0, stream>>>(p);
     return cudaGetLastError();
+}
+
+template <int kMode>
+cudaError_t launch_mode(const SimParams& p, int blocks, cudaStream_t stream)
+{
+    switch (sim_group_width(p.n_pre + p.n_dec)) {
+    case 4: return launch_width<4, kMode>(p, blocks, stream);
+    case 8: return launch_width<8, kMode>(p, blocks, stream);
+    case 16: return launch_width<16, kMode>(p, blocks, stream);
+    default: return launch_width<32, kMode>(p, blocks, stream);
+    }
 }
 
 }  // namespace
@@ -851,20 +865,11 @@ cudaError_t launch_width(const SimParams& p, int blocks, cudaStream_t stream)
 cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
 {
     (void)warps_per_block;
-    bool ext = false;  // the proxy's signals or batched prefill
-    for (int i = 0; i < p.n_sets; ++i) ext = ext || p.sets[i].proxy != 0 || p.sets[i].poll_us > 0;
-    ext = ext || p.pre_batch > 0;
-    cudaError_t e;
-    switch (sim_group_width(p.n_pre + p.n_dec) * 2 + (ext ? 1 : 0)) {
-    case 8: e = launch_width<4, false>(p, blocks, stream); break;
-    case 9: e = launch_width<4, true>(p, blocks, stream); break;
-    case 16: e = launch_width<8, false>(p, blocks, stream); break;
-    case 17: e = launch_width<8, true>(p, blocks, stream); break;
-    case 32: e = launch_width<16, false>(p, blocks, stream); break;
-    case 33: e = launch_width<16, true>(p, blocks, stream); break;
-    case 64: e = launch_width<32, false>(p, blocks, stream); break;
-    default: e = launch_width<32, true>(p, blocks, stream); break;
-    }
+    bool signals = false;  // the proxy's ledger backlog or polled occupancy in some constant set
+    for (int i = 0; i < p.n_sets; ++i) signals = signals || p.sets[i].proxy != 0 || p.sets[i].poll_us > 0;
+    const cudaError_t e = p.pre_batch > 0 ? launch_mode<2>(p, blocks, stream)
+                          : signals       ? launch_mode<1>(p, blocks, stream)
+                                          : launch_mode<0>(p, blocks, stream);
     if (e != cudaSuccess) return e;
     if (p.n_rows > 0) {
         const int64_t hb = p.n_rows < (int64_t)blocks * 8 ? p.n_rows : (int64_t)blocks * 8;
