@@ -8,16 +8,18 @@
 // a_d^s + m_d^s * o_hat with a_d^s = sigma_s w_b backlog_d + w_q A_d and
 // m_d^s = sigma_s w_s tau_dec rho kappa_d >= 0.  Each block stages the
 // instance state into shared memory with a TMA bulk copy (cp.async.bulk +
-// mbarrier) while its first request vectors are already in flight, builds the
-// four per-class envelopes (one thread per (class, line): a division-free
-// Pareto test -- a line with both a larger intercept and a larger slope than
-// another can never win -- then, for the few surviving lines, the interval of
-// o_hat on which the line wins and its rank), and streams requests with
-// 128-bit loads, software-pipelined one vector ahead: a binary search over the
-// envelope's breakpoints gives the argmin, whose fp32 cost is then evaluated
-// from the full formula.  The work per request is O(log envelope size) instead
-// of O(instances), which keeps the kernel on the HBM roofline.  One block per
-// SM, so the envelope is built 152 times, not once per request tile.
+// mbarrier) while its first request vectors are already in flight, then builds
+// the four per-class envelopes: for pools of up to 64 instances one warp per
+// class walks the envelope from o_hat = 0 by gift wrapping (one warp argmin
+// per segment); wider pools use every thread (a Pareto test, the o_hat
+// interval on which each surviving line wins, and its rank).  Each segment
+// keeps its instance's cost terms in one 16-byte entry.  Requests stream with
+// 128-bit loads, software-pipelined two vectors ahead: the count of
+// breakpoints at or below o_hat (a binary search past 8 segments) gives the
+// argmin, whose fp32 cost is then evaluated from the full formula.  The work
+// per request is O(log envelope size) instead of O(instances), which keeps the
+// kernel on the HBM roofline.  One block per SM, so the envelope is built 152
+// times, not once per request tile.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -39,7 +41,7 @@ struct __align__(16) Smem {
     int valid_tmp[4][kMaxInst];
     int pareto[4][kMaxInst];
     float seg_lo[4][kMaxInst];
-    int seg_id[4][kMaxInst];
+    float4 seg_e[4][kMaxInst];  // per segment: kappa, BK, WQA of its instance, and the index (as bits)
     float4 brk[4][2];  // breakpoints 1..7 of each class (seg_lo[s][1..7]), +inf past the last
     int nseg[4];
     unsigned long long bar;
@@ -89,28 +91,37 @@ __device__ __forceinline__ ReqTerms req_terms(const ScoreParams& P, float p, flo
     return ReqTerms{g, toh * P.c[3]};
 }
 
-__device__ __forceinline__ float cost_at(const Smem& sm, const ScoreParams& P, ReqTerms r, int s, int d)
+// the full cost at the segment's instance e = (kappa_d, BK_d, WQA_d, d)
+__device__ __forceinline__ float cost_at(const ScoreParams& P, ReqTerms r, int s, float4 e)
 {
-    const float own = fmaf(r.h, sm.kap[d], r.g);
-    return fmaf(P.c[9 + s], fmaf(P.c[1], own, sm.bk[d]), sm.wqa[d]);
+    const float own = fmaf(r.h, e.x, r.g);
+    return fmaf(P.c[9 + s], fmaf(P.c[1], own, e.y), e.z);
 }
 
+// the segment entry of instance d
+__device__ __forceinline__ float4 seg_entry(const Smem& sm, const ScoreParams& P, int d)
+{
+    const float A = sm.a[d];
+    return make_float4(sm.kap[d], P.c[0] * fmaf(P.c[5], sm.q[d], P.c[7] * A), P.c[2] * A, __int_as_float(d));
+}
+
+// wide: some class has more than 8 segments (block-uniform), so the segment is
+// found by binary search instead of the branch-free count over 8 breakpoints
 __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, float p, float oh, uint32_t s,
-                                          int& arg, float& cost)
+                                          bool wide, int& arg, float& cost)
 {
     if (s >= 4) {
         arg = -1;
         cost = __int_as_float(0x7fc00000);
         return;
     }
-    const int ns = sm.nseg[s];
     int seg;
-    if (ns <= 8) {  // segments start at 0 and at the sorted breakpoints: count those <= o_hat
+    if (!wide) {  // segments start at 0 and at the sorted breakpoints: count those <= o_hat
         const float4 b0 = sm.brk[s][0], b1 = sm.brk[s][1];
         seg = (int)(b0.x <= oh) + (int)(b0.y <= oh) + (int)(b0.z <= oh) + (int)(b0.w <= oh) + (int)(b1.x <= oh) +
               (int)(b1.y <= oh) + (int)(b1.z <= oh);
     } else {
-        int lo = 0, span = ns;
+        int lo = 0, span = sm.nseg[s];
         while (span > 1) {  // last segment whose left end is <= o_hat
             const int half = span >> 1;
             if (sm.seg_lo[s][lo + half] <= oh) lo += half;
@@ -118,9 +129,9 @@ __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, 
         }
         seg = lo;
     }
-    const int d = sm.seg_id[s][seg];
-    arg = d;
-    cost = cost_at(sm, P, req_terms(P, p, oh), (int)s, d);
+    const float4 e = sm.seg_e[s][seg];
+    arg = __float_as_int(e.w);
+    cost = cost_at(P, req_terms(P, p, oh), (int)s, e);
 }
 
 // (intercept, slope, index) lexicographic order of envelope lines
@@ -129,120 +140,108 @@ __device__ __forceinline__ bool line_less(float a, float m, int i, float b, floa
     return a < b || (a == b && (m < n || (m == n && i < j)));
 }
 
-// Lower envelope of one class's lines with one warp, for up to 64 lines:
-// a bitonic sort by (intercept, slope, index) across the lanes (two lines per
-// lane), an exclusive prefix minimum of the slopes that keeps the Pareto
-// lines (those whose slope is below every line sorted before them), and the
-// convex-hull stack pass over the survivors by lane 0, which writes the
-// segments' left ends and lines.
-__device__ void warp_envelope(Smem& sm, int s, int n_inst, int lane)
+// lexicographic (x, m, i) minimum over the warp; every lane gets the result
+__device__ __forceinline__ void warp_min_xmi(float& x, float& m, int& i)
 {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float px = __shfl_xor_sync(0xffffffffu, x, off);
+        const float pm = __shfl_xor_sync(0xffffffffu, m, off);
+        const int pi = __shfl_xor_sync(0xffffffffu, i, off);
+        if (line_less(px, pm, pi, x, m, i)) {
+            x = px;
+            m = pm;
+            i = pi;
+        }
+    }
+}
+
+// Lower envelope of one class's lines over o_hat >= 0 with one warp, for up to
+// 64 lines (two per lane), by gift wrapping: the first segment's line is the
+// least (intercept, slope, index); from the current line the next one is,
+// among the lines of smaller slope, the one whose crossing with it comes first
+// (ties: smaller slope, then lower index), and the crossing is that segment's
+// left end.  Each step lowers the slope, so the loop ends within n_inst steps,
+// one warp argmin each (a handful for the states seen in practice: the
+// envelope of n random lines has O(log n) segments).  Left ends are kept
+// non-decreasing against rounding.  Segment t stays in lane t % 32, slot
+// t / 32, until the warp writes the segment arrays and the padded breakpoints.
+__device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst, int lane)
+{
+    const float inf = __int_as_float(0x7f800000);
+    constexpr int kNone = 1 << 20;
+    const float sig = P.c[9 + s];
+    const float ks = sig * P.c[1] * P.c[6] * P.c[3];
     float a[2], m[2];
-    int id[2];
+    bool live[2];
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
+    for (int r = 0; r < 2; ++r) {  // the line of instance j (the expression line_of evaluates)
         const int j = lane + 32 * r;
-        const bool real = j < n_inst;
-        a[r] = real ? sm.la[s][j] : __int_as_float(0x7f800000);
-        m[r] = real ? sm.lm[s][j] : __int_as_float(0x7f800000);
-        id[r] = real ? j : 1 << 20;
+        const float A = j < n_inst ? sm.a[j] : 0.0f;
+        a[r] = j < n_inst ? fmaf(sig, P.c[0] * fmaf(P.c[5], sm.q[j], P.c[7] * A), P.c[2] * A) : inf;
+        m[r] = j < n_inst ? ks * sm.kap[j] : inf;
+        // a non-finite line (outside the input contract) takes no part, which keeps
+        // every comparison below a total order and the warp's decisions uniform
+        live[r] = fabsf(a[r]) < inf && fabsf(m[r]) < inf;
+        if (!live[r]) a[r] = m[r] = inf;
     }
+    float ca = a[0], cm = m[0];
+    int ci = live[0] ? lane : kNone;
+    if (live[1] && line_less(a[1], m[1], lane + 32, ca, cm, ci)) {
+        ca = a[1];
+        cm = m[1];
+        ci = lane + 32;
+    }
+    warp_min_xmi(ca, cm, ci);
+    if (ci == kNone) ci = 0;  // no finite line at all (outside the input contract)
+    float lo0 = 0.0f, lo1 = 0.0f;
+    int id0 = ci, id1 = 0;
+    float x_cur = 0.0f;
+    int nseg = 1;
+    while (nseg < n_inst) {
+        float bx = inf, bm = inf;
+        int bi = kNone;
 #pragma unroll
-    for (int k = 2; k <= 64; k <<= 1) {
-#pragma unroll
-        for (int jj = k >> 1; jj > 0; jj >>= 1) {
-            if (jj == 32) {  // partner in the same lane, other slot
-                const bool asc = (lane & k) == 0;  // element index lane has bit 5 clear
-                const bool sw = asc == line_less(a[1], m[1], id[1], a[0], m[0], id[0]);
-                if (sw) {
-                    float t = a[0]; a[0] = a[1]; a[1] = t;
-                    t = m[0]; m[0] = m[1]; m[1] = t;
-                    const int u = id[0]; id[0] = id[1]; id[1] = u;
+        for (int r = 0; r < 2; ++r) {
+            const int j = lane + 32 * r;
+            if (live[r] && m[r] < cm) {
+                const float x = (a[r] - ca) / (cm - m[r]);
+                if (x == x && line_less(x, m[r], j, bx, bm, bi)) {
+                    bx = x;
+                    bm = m[r];
+                    bi = j;
                 }
+            }
+        }
+        warp_min_xmi(bx, bm, bi);
+        if (bi == kNone) break;  // warp-uniform: no line of smaller slope is left
+        ca = __shfl_sync(0xffffffffu, bi < 32 ? a[0] : a[1], bi & 31);
+        cm = bm;
+        x_cur = fmaxf(bx, x_cur);
+        if (lane == (nseg & 31)) {
+            if (nseg < 32) {
+                lo0 = x_cur;
+                id0 = bi;
             } else {
-#pragma unroll
-                for (int r = 0; r < 2; ++r) {
-                    const int j = lane + 32 * r;
-                    const float pa = __shfl_xor_sync(0xffffffffu, a[r], jj);
-                    const float pm = __shfl_xor_sync(0xffffffffu, m[r], jj);
-                    const int pi = __shfl_xor_sync(0xffffffffu, id[r], jj);
-                    const bool asc = (j & k) == 0;
-                    const bool lower = (j & jj) == 0;  // this element takes the smaller key when ascending
-                    const bool p_less = line_less(pa, pm, pi, a[r], m[r], id[r]);
-                    if (lower == asc ? p_less : !p_less) {
-                        a[r] = pa;
-                        m[r] = pm;
-                        id[r] = pi;
-                    }
-                }
+                lo1 = x_cur;
+                id1 = bi;
             }
         }
+        ++nseg;
     }
-    // exclusive prefix minimum of the slopes in sorted order (element j = lane + 32 r)
-    float incl0 = m[0];
-    for (int off = 1; off < 32; off <<= 1) {
-        const float v = __shfl_up_sync(0xffffffffu, incl0, off);
-        if (lane >= off) incl0 = fminf(incl0, v);
+    if (lane < nseg) {
+        sm.seg_lo[s][lane] = lo0;
+        sm.seg_e[s][lane] = seg_entry(sm, P, id0);
     }
-    const float all0 = __shfl_sync(0xffffffffu, incl0, 31);
-    float excl0 = __shfl_up_sync(0xffffffffu, incl0, 1);
-    if (lane == 0) excl0 = __int_as_float(0x7f800000);
-    float incl1 = m[1];
-    for (int off = 1; off < 32; off <<= 1) {
-        const float v = __shfl_up_sync(0xffffffffu, incl1, off);
-        if (lane >= off) incl1 = fminf(incl1, v);
+    if (lane + 32 < nseg) {
+        sm.seg_lo[s][lane + 32] = lo1;
+        sm.seg_e[s][lane + 32] = seg_entry(sm, P, id1);
     }
-    float excl1 = __shfl_up_sync(0xffffffffu, incl1, 1);
-    excl1 = lane == 0 ? all0 : fminf(excl1, all0);
-    const bool par0 = id[0] < (1 << 20) && m[0] < excl0;
-    const bool par1 = id[1] < (1 << 20) && m[1] < excl1;
-    // compact the Pareto lines, in sorted order, into the segment arrays as scratch
-    const uint32_t b0 = __ballot_sync(0xffffffffu, par0), b1 = __ballot_sync(0xffffffffu, par1);
-    const uint32_t below = (1u << lane) - 1u;
-    if (par0) {
-        const int pos = __popc(b0 & below);
-        sm.lo_tmp[s][pos] = a[0];
-        sm.seg_lo[s][pos] = m[0];
-        sm.valid_tmp[s][pos] = id[0];
+    if (lane >= 1 && lane <= 8) {  // padded breakpoints for the branch-free segment count
+        float* b = reinterpret_cast<float*>(&sm.brk[s][0]);
+        b[lane - 1] = lane < nseg ? lo0 : inf;
     }
-    if (par1) {
-        const int pos = __popc(b0) + __popc(b1 & below);
-        sm.lo_tmp[s][pos] = a[1];
-        sm.seg_lo[s][pos] = m[1];
-        sm.valid_tmp[s][pos] = id[1];
-    }
-    __syncwarp();
-    if (lane == 0) {  // lower hull: slopes strictly decrease, intercepts strictly increase
-        const int np = __popc(b0) + __popc(b1);
-        int top = 0;  // stack kept in place at the front of the scratch arrays
-        for (int t = 0; t < np; ++t) {
-            const float at = sm.lo_tmp[s][t], mt = sm.seg_lo[s][t];
-            const int it = sm.valid_tmp[s][t];
-            while (top >= 2) {
-                const float a1 = sm.lo_tmp[s][top - 2], m1 = sm.seg_lo[s][top - 2];
-                const float a2 = sm.lo_tmp[s][top - 1], m2 = sm.seg_lo[s][top - 1];
-                // the previous top wins nowhere if the new line meets the one below it no later
-                // (at - a1) / (m1 - mt) <= (a2 - a1) / (m1 - m2), denominators positive
-                if ((at - a1) * (m1 - m2) <= (a2 - a1) * (m1 - mt)) --top;
-                else break;
-            }
-            sm.lo_tmp[s][top] = at;
-            sm.seg_lo[s][top] = mt;
-            sm.valid_tmp[s][top] = it;
-            ++top;
-        }
-        // segment t covers o_hat from the crossing of lines t-1 and t
-        float prev_a = 0.0f, prev_m = 0.0f;
-        for (int t = 0; t < top; ++t) {
-            const float at = sm.lo_tmp[s][t], mt = sm.seg_lo[s][t];
-            const int it = sm.valid_tmp[s][t];
-            sm.seg_lo[s][t] = t == 0 ? 0.0f : (at - prev_a) / (prev_m - mt);
-            sm.seg_id[s][t] = it;
-            prev_a = at;
-            prev_m = mt;
-        }
-        sm.nseg[s] = top;
-    }
+    if (lane == 0) sm.nseg[s] = nseg;
 }
 
 template <bool kVec>
@@ -327,112 +326,112 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         }
     }
     __syncthreads();
-    for (int d = tid; d < n_inst; d += kThreads) {
-        sm.bk[d] = P.c[0] * fmaf(P.c[5], sm.q[d], P.c[7] * sm.a[d]);
-        sm.wqa[d] = P.c[2] * sm.a[d];
-    }
-    __syncthreads();
-
-    // ---- per-class lower envelope
-    for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {
-        const int s = idx / n_inst, d = idx - s * n_inst;
-        line_of(sm, P, s, d, sm.la[s][d], sm.lm[s][d]);
-    }
-    if (tid < 4) sm.nseg[tid] = 0;
-    __syncthreads();
-    if (n_inst <= 64) {
-        if (tid < 128) warp_envelope(sm, tid >> 5, n_inst, tid & 31);  // one warp per class
+    if (n_inst <= 64) {  // warps 0-3 build the four class envelopes from the staged state
+        if (tid < 128) warp_envelope(sm, P, tid >> 5, n_inst, tid & 31);
         __syncthreads();
     } else {
+        for (int d = tid; d < n_inst; d += kThreads) {
+            sm.bk[d] = P.c[0] * fmaf(P.c[5], sm.q[d], P.c[7] * sm.a[d]);
+            sm.wqa[d] = P.c[2] * sm.a[d];
+        }
+        __syncthreads();
+        // ---- per-class lower envelope over all lines
+        for (int idx = tid; idx < 4 * n_inst; idx += kThreads) {
+            const int s = idx / n_inst, d = idx - s * n_inst;
+            line_of(sm, P, s, d, sm.la[s][d], sm.lm[s][d]);
+        }
+        if (tid < 4) sm.nseg[tid] = 0;
+        __syncthreads();
         // wider pools: each (class, line) pair is handled by tpp threads that
         // split its scans over the other lines and combine them with butterfly
         // shuffles, so all 32 warps of the block share the O(n^2) work
-    int tpp = kThreads / (4 * n_inst);  // threads per pair: a power of two in [1, 32]
-    tpp = tpp >= 32 ? 32 : tpp >= 16 ? 16 : tpp >= 8 ? 8 : tpp >= 4 ? 4 : tpp >= 2 ? 2 : 1;
-    const int pair = tid / tpp, part = tid - pair * tpp;
-    const bool act = pair < 4 * n_inst;
-    const int es = act ? pair / n_inst : 0;
-    const int ed = act ? pair - es * n_inst : 0;
-    const float ad = sm.la[es][ed], md = sm.lm[es][ed];
-    // Pareto filter: a line with a smaller-or-equal intercept and slope (ties: lowest index) hides it
-    bool dominated = false;
-    if (act) {
+        int tpp = kThreads / (4 * n_inst);  // threads per pair: a power of two in [1, 32]
+        tpp = tpp >= 32 ? 32 : tpp >= 16 ? 16 : tpp >= 8 ? 8 : tpp >= 4 ? 4 : tpp >= 2 ? 2 : 1;
+        const int pair = tid / tpp, part = tid - pair * tpp;
+        const bool act = pair < 4 * n_inst;
+        const int es = act ? pair / n_inst : 0;
+        const int ed = act ? pair - es * n_inst : 0;
+        const float ad = sm.la[es][ed], md = sm.lm[es][ed];
+        // Pareto filter: a line with a smaller-or-equal intercept and slope (ties: lowest index) hides it
+        bool dominated = false;
+        if (act) {
 #pragma unroll 4
-        for (int e = part; e < n_inst; e += tpp) {
-            const float ae = sm.la[es][e], me = sm.lm[es][e];
-            dominated |= ae <= ad && me <= md && (ae < ad || me < md || e < ed);
-        }
-    }
-    for (int off = 1; off < tpp; off <<= 1) dominated |= __shfl_xor_sync(0xffffffffu, dominated, off, tpp);
-    if (act && part == 0) sm.pareto[es][ed] = !dominated;
-    __syncthreads();
-    // the o_hat interval on which a surviving line wins
-    const bool cand = act && sm.pareto[es][ed];
-    float lo = 0.0f, hi = __int_as_float(0x7f800000);
-    if (cand) {
-#pragma unroll 4
-        for (int e = part; e < n_inst; e += tpp) {
-            if (e == ed || !sm.pareto[es][e]) continue;
-            const float ae = sm.la[es][e], me = sm.lm[es][e];
-            if (me > md) {
-                lo = fmaxf(lo, (ad - ae) / (me - md));
-            } else if (me < md) {
-                hi = fminf(hi, (ae - ad) / (md - me));
+            for (int e = part; e < n_inst; e += tpp) {
+                const float ae = sm.la[es][e], me = sm.lm[es][e];
+                dominated |= ae <= ad && me <= md && (ae < ad || me < md || e < ed);
             }
         }
-    }
-    for (int off = 1; off < tpp; off <<= 1) {
-        lo = fmaxf(lo, __shfl_xor_sync(0xffffffffu, lo, off, tpp));
-        hi = fminf(hi, __shfl_xor_sync(0xffffffffu, hi, off, tpp));
-    }
-    const bool valid = cand && lo < hi;
-    if (act && part == 0) {
-        sm.valid_tmp[es][ed] = valid;
-        sm.lo_tmp[es][ed] = lo;
-    }
-    __syncthreads();
-    // rank of each winning interval by its left end
-    int rank = 0;
-    if (valid) {
+        for (int off = 1; off < tpp; off <<= 1) dominated |= __shfl_xor_sync(0xffffffffu, dominated, off, tpp);
+        if (act && part == 0) sm.pareto[es][ed] = !dominated;
+        __syncthreads();
+        // the o_hat interval on which a surviving line wins
+        const bool cand = act && sm.pareto[es][ed];
+        float lo = 0.0f, hi = __int_as_float(0x7f800000);
+        if (cand) {
 #pragma unroll 4
-        for (int e = part; e < n_inst; e += tpp) {
-            const float le = sm.lo_tmp[es][e];
-            rank += sm.valid_tmp[es][e] && (le < lo || (le == lo && e < ed));
-        }
-    }
-    for (int off = 1; off < tpp; off <<= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off, tpp);
-    if (valid && part == 0) {
-        sm.seg_lo[es][rank] = lo;
-        sm.seg_id[es][rank] = ed;
-        atomicAdd(&sm.nseg[es], 1);
-    }
-    __syncthreads();
-    }
-    if (tid < 4 && sm.nseg[tid] == 0) {  // rounding left no winner (never with finite inputs): brute force line
-        int best = 0;
-        float bv = 0.0f;
-        for (int d = 0; d < n_inst; ++d) {
-            float a, m;
-            line_of(sm, P, tid, d, a, m);
-            if (d == 0 || a < bv) {
-                bv = a;
-                best = d;
+            for (int e = part; e < n_inst; e += tpp) {
+                if (e == ed || !sm.pareto[es][e]) continue;
+                const float ae = sm.la[es][e], me = sm.lm[es][e];
+                if (me > md) {
+                    lo = fmaxf(lo, (ad - ae) / (me - md));
+                } else if (me < md) {
+                    hi = fminf(hi, (ae - ad) / (md - me));
+                }
             }
         }
-        sm.seg_lo[tid][0] = 0.0f;
-        sm.seg_id[tid][0] = best;
-        sm.nseg[tid] = 1;
-    }
-    __syncthreads();
+        for (int off = 1; off < tpp; off <<= 1) {
+            lo = fmaxf(lo, __shfl_xor_sync(0xffffffffu, lo, off, tpp));
+            hi = fminf(hi, __shfl_xor_sync(0xffffffffu, hi, off, tpp));
+        }
+        const bool valid = cand && lo < hi;
+        if (act && part == 0) {
+            sm.valid_tmp[es][ed] = valid;
+            sm.lo_tmp[es][ed] = lo;
+        }
+        __syncthreads();
+        // rank of each winning interval by its left end
+        int rank = 0;
+        if (valid) {
+#pragma unroll 4
+            for (int e = part; e < n_inst; e += tpp) {
+                const float le = sm.lo_tmp[es][e];
+                rank += sm.valid_tmp[es][e] && (le < lo || (le == lo && e < ed));
+            }
+        }
+        for (int off = 1; off < tpp; off <<= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off, tpp);
+        if (valid && part == 0) {
+            sm.seg_lo[es][rank] = lo;
+            sm.seg_e[es][rank] = seg_entry(sm, P, ed);
+            atomicAdd(&sm.nseg[es], 1);
+        }
+        __syncthreads();
+        if (tid < 4 && sm.nseg[tid] == 0) {  // rounding left no winner (never with finite inputs): brute force line
+            int best = 0;
+            float bv = 0.0f;
+            for (int d = 0; d < n_inst; ++d) {
+                float a, m;
+                line_of(sm, P, tid, d, a, m);
+                if (d == 0 || a < bv) {
+                    bv = a;
+                    best = d;
+                }
+            }
+            sm.seg_lo[tid][0] = 0.0f;
+            sm.seg_e[tid][0] = seg_entry(sm, P, best);
+            sm.nseg[tid] = 1;
+        }
+        __syncthreads();
 
-    if (tid < 4 * 8) {  // padded breakpoints for the branch-free segment count
-        const int cs = tid >> 3, t = (tid & 7) + 1;
-        float* b = reinterpret_cast<float*>(&sm.brk[cs][0]);
-        b[t - 1] = t < sm.nseg[cs] ? sm.seg_lo[cs][t] : __int_as_float(0x7f800000);
+        if (tid < 4 * 8) {  // padded breakpoints for the branch-free segment count
+            const int cs = tid >> 3, t = (tid & 7) + 1;
+            float* b = reinterpret_cast<float*>(&sm.brk[cs][0]);
+            b[t - 1] = t < sm.nseg[cs] ? sm.seg_lo[cs][t] : __int_as_float(0x7f800000);
+        }
+        __syncthreads();
     }
-    __syncthreads();
 
     // ---- stream the requests (the first vector was loaded before the prologue)
+    const bool wide = sm.nseg[0] > 8 || sm.nseg[1] > 8 || sm.nseg[2] > 8 || sm.nseg[3] > 8;
     if (kVec) {
         int4* a4 = reinterpret_cast<int4*>(P.argmin);
         float4* f4 = reinterpret_cast<float4*>(P.cost);
@@ -448,10 +447,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
             }
             int4 ai;
             float4 fc;
-            score_one(sm, P, pv.x, ov.x, cv & 0xFFu, ai.x, fc.x);
-            score_one(sm, P, pv.y, ov.y, (cv >> 8) & 0xFFu, ai.y, fc.y);
-            score_one(sm, P, pv.z, ov.z, (cv >> 16) & 0xFFu, ai.z, fc.z);
-            score_one(sm, P, pv.w, ov.w, cv >> 24, ai.w, fc.w);
+            score_one(sm, P, pv.x, ov.x, cv & 0xFFu, wide, ai.x, fc.x);
+            score_one(sm, P, pv.y, ov.y, (cv >> 8) & 0xFFu, wide, ai.y, fc.y);
+            score_one(sm, P, pv.z, ov.z, (cv >> 16) & 0xFFu, wide, ai.z, fc.z);
+            score_one(sm, P, pv.w, ov.w, cv >> 24, wide, ai.w, fc.w);
             __stcs(a4 + v, ai);
             __stcs(f4 + v, fc);
             v += stride;
@@ -468,7 +467,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
             const int64_t i = (nv << 2) + tid;
             int ai;
             float fc;
-            score_one(sm, P, P.p[i], P.oh[i], P.cls[i], ai, fc);
+            score_one(sm, P, P.p[i], P.oh[i], P.cls[i], wide, ai, fc);
             P.argmin[i] = ai;
             P.cost[i] = fc;
         }
@@ -476,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         for (int64_t i = (int64_t)blockIdx.x * kThreads + tid; i < P.n; i += (int64_t)gridDim.x * kThreads) {
             int ai;
             float fc;
-            score_one(sm, P, P.p[i], P.oh[i], P.cls[i], ai, fc);
+            score_one(sm, P, P.p[i], P.oh[i], P.cls[i], wide, ai, fc);
             P.argmin[i] = ai;
             P.cost[i] = fc;
         }

@@ -106,6 +106,29 @@ def test_degenerate_states(orc):
     _check(orc, p, oh, cls, Q, A, kap, zero_rho, am, cost)
 
 
+@pytest.mark.parametrize("n_inst", [9, 33, 64, 65, 130])
+def test_every_line_on_the_envelope(orc, n_inst):
+    """A state whose lower envelope holds every instance (queued tokens convex in
+    the index, KV occupancy falling linearly): breakpoints at about 23 (2d + 1)
+    tokens of o_hat, so the requests cross every segment, past the branch-free
+    count of 8 segments and past 32 (the second register slot of the warp
+    walk), and through the all-thread path for wider pools."""
+    ctr = need_gpu()
+    d = np.arange(n_inst)
+    Q = (37.0 * d * d * (64.0 / n_inst) ** 2).astype(np.float32)
+    A = np.zeros(n_inst, np.float32)
+    kap = ((n_inst - d) / n_inst).astype(np.float32)
+    n = 20_000
+    rng = np.random.default_rng(n_inst)
+    oh = np.floor(rng.random(n) * 3300.0).astype(np.float32)
+    p = np.floor(rng.random(n) * 4000.0 + 16.0).astype(np.float32)
+    cls = rng.integers(0, 4, n).astype(np.uint8)
+    ref_am, _, _ = orc.score_batch(p, oh, cls, Q, A, kap, W.SCORE_CONSTS)
+    assert np.unique(ref_am).size >= n_inst - 1  # the case exercises what it claims
+    am, cost = _run(ctr, p, oh, cls, Q, A, kap, W.SCORE_CONSTS)
+    _check(orc, p, oh, cls, Q, A, kap, W.SCORE_CONSTS, am, cost)
+
+
 def test_hand_computed_exact(orc):
     ctr = need_gpu()
     with open(os.path.join(GOLDEN, "score_hand.json")) as f:
