@@ -146,6 +146,7 @@ def run_reference(args, rank, world):
 
 # ---------------------------------------------------------------- GPU arm
 SIM_SOURCES = ("paper_2609_16206_gb300/csrc/sim.cu", "paper_2609_16206_gb300/csrc/ctr_internal.cuh", "include/ctr.h")
+SCORE_SOURCES = ("paper_2609_16206_gb300/csrc/score.cu", "paper_2609_16206_gb300/csrc/ctr_internal.cuh", "include/ctr.h")
 
 
 def _strip_comments(src: str) -> str:
@@ -172,10 +173,10 @@ def _strip_comments(src: str) -> str:
     return "\n".join(line.rstrip() for line in "".join(out).splitlines() if line.strip())
 
 
-def _source_hash() -> str:
-    """Hash of the code (comments stripped) of the files that define the simulator kernel."""
+def _source_hash(sources=SIM_SOURCES) -> str:
+    """Hash of the code (comments stripped) of the files that define a kernel (the simulator's by default)."""
     h = hashlib.sha256()
-    for rel in SIM_SOURCES:
+    for rel in sources:
         with open(os.path.join(ROOT, rel), encoding="utf-8") as f:
             h.update(rel.encode() + _strip_comments(f.read()).encode())
     return h.hexdigest()[:16]
@@ -441,10 +442,13 @@ def run_ours(args, rank, world, local_rank):
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     score_bytes = 17 * N_SCORE_REQ + 3 * 4 * N_SCORE_INST
     pairs_per_s = N_SCORE_REQ * N_SCORE_INST / (rot_ms / 1e3)  # graph-batched launches, inputs from HBM
+    score_dram = SCORE_DRAM_PER_LAUNCH.get(_source_hash(SCORE_SOURCES))
     score_roof = {"bound": "hbm", "unit": "GB/s", "achieved": score_bytes / (rot_ms / 1e3) / 1e9,
-                  "peak": hbm, "traffic": 9.50e6, "launch_ms": rot_ms, "launch_ms_in_step": per_kernel_ms["score"],
-                  "traffic_note": "ncu DRAM read 9.50 MB, write 0 B within one graph launch (the 8.4 MB of outputs "
-                                  "are written back from L2 after it)",
+                  "peak": hbm, "traffic": None if score_dram is None else score_dram["read"] + score_dram["write"],
+                  "launch_ms": rot_ms, "launch_ms_in_step": per_kernel_ms["score"],
+                  "traffic_note": "no counters for this kernel source" if score_dram is None else
+                  f"ncu DRAM read {score_dram['read'] / 1e6:.2f} MB, write {score_dram['write'] / 1e6:.2f} MB in "
+                  "one launch of the step (the outputs are written back from L2 after it)",
                   "timing": f"{rot_sets} buffer sets ({rot_sets * score_bytes / 1e6:.0f} MB, > 4x L2) back to back "
                             f"from one CUDA graph, x{g_reps}; outputs identical across sets: {rot_ok}"}
     score_roof["frac"] = score_roof["achieved"] / hbm
@@ -487,6 +491,11 @@ def run_ours(args, rank, world, local_rank):
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
     "ba5dc650cdbd67a7": {"warp_inst": 164340141282, "dram_bytes": 30.62e9 + 20.48e9},
+}
+
+SCORE_DRAM_PER_LAUNCH: dict = {
+    # 2^20 requests x 64 instances, one launch inside the step (profiles/score_kernel_standalone_2p20x64.md)
+    "0cf447425ccfdb3c": {"read": 9.485e6, "write": 0.0},
 }
 
 
