@@ -490,12 +490,12 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "ba5dc650cdbd67a7": {"warp_inst": 164340141282, "dram_bytes": 30.62e9 + 20.48e9},
+    "7e70a5fe20c12da0": {"warp_inst": 156907495617, "dram_bytes": 30.61e9 + 20.29e9},
 }
 
 SCORE_DRAM_PER_LAUNCH: dict = {
     # 2^20 requests x 64 instances, one launch inside the step (profiles/score_kernel_standalone_2p20x64.md)
-    "0cf447425ccfdb3c": {"read": 9.485e6, "write": 0.0},
+    "6e38b5261e3bff8b": {"read": 9.49e6, "write": 0.0},
 }
 
 

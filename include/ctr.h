@@ -35,6 +35,7 @@ extern "C" {
 #define CTR_MAX_CLASSES 4         /* SLO classes */
 #define CTR_MAX_CONST_SETS 128    /* cost-constant sets per ctr_simulate call */
 #define CTR_MAX_REQUESTS (1 << 23) /* requests per replica */
+#define CTR_MAX_STEPS_PER_INSTANCE ((1LL << 31) - (1LL << 21)) /* bound on the decode-step budget */
 #define CTR_SCORE_N_CONST 13      /* length of the standalone scorer's constant vector */
 #define CTR_SCORE_MAX_INST 256    /* instances per standalone scoring call */
 
@@ -120,7 +121,7 @@ typedef struct ctr_sim_cfg {
     int32_t heuristic_threshold_tokens; /* length heuristic: o_hat >= threshold uses predicted-token load */
     int64_t ttft_slo_us[4];           /* per class, >= 0 */
     int64_t tpot_slo_us[4];
-    int64_t max_steps_per_instance;   /* decode-step budget per instance and row, >= 1 */
+    int64_t max_steps_per_instance;   /* decode-step budget per instance and row, 1..CTR_MAX_STEPS_PER_INSTANCE */
     int32_t cap_pending;              /* requests routed to a decode instance whose KV is not ready, 1..2^20 */
     int32_t cap_waiting;              /* KV-ready requests not yet admitted, 1..2^20 */
     int32_t cap_active;               /* decode batch size, 1..2^20 */
@@ -247,7 +248,8 @@ int ctr_goodput(const ctr_sim_cfg* cfg /* host */, ctr_requests trace, int32_t n
 /* ctr_strerror -- static description of a CTR_* code. */
 const char* ctr_strerror(int code);
 
-/* ctr_abi_version -- increments on any change to the structs or signatures. */
+/* ctr_abi_version -- increments on any change to the structs, the signatures or
+ * the accepted ranges. */
 int ctr_abi_version(void);
 
 #ifdef __cplusplus

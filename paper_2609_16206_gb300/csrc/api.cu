@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 4;
+constexpr int kAbiVersion = 5;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -36,7 +36,7 @@ bool valid_sim_cfg(const ctr_sim_cfg* c)
     if (c->heuristic_threshold_tokens < 0) return false;
     for (int i = 0; i < CTR_MAX_CLASSES; ++i)
         if (c->ttft_slo_us[i] < 0 || c->tpot_slo_us[i] < 0) return false;
-    if (c->max_steps_per_instance < 1) return false;
+    if (!in_range(c->max_steps_per_instance, 1, CTR_MAX_STEPS_PER_INSTANCE)) return false;
     if (!in_range(c->prefill_batch_tokens, 0, 1LL << 30)) return false;
     const int64_t cap_max = 1LL << 20;
     if (!in_range(c->cap_pending, 1, cap_max) || !in_range(c->cap_waiting, 1, cap_max) ||

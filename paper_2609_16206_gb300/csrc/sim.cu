@@ -110,10 +110,15 @@ __device__ __forceinline__ int64_t floor_div_small(int64_t x, int64_t d)
     return q;
 }
 
-// floor(x / kv_div) for 0 <= x < 2^32 with magic = ceil(2^64 / kv_div), exact
+// floor(x / kv_div) for 0 <= x < 2^32 with magic = ceil(2^64 / kv_div), exact: the
+// 96-bit product x * magic shifted right by 64, from two 32 x 32-bit products
 __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
 {
-    return P.kv_div == 1 ? x : (int64_t)__umul64hi((uint64_t)x, P.kv_div_magic);
+    if (P.kv_div == 1) return x;
+    const uint32_t xl = (uint32_t)x;
+    const uint64_t lo = (uint64_t)xl * (uint32_t)P.kv_div_magic;
+    const uint64_t hi = (uint64_t)xl * (uint32_t)(P.kv_div_magic >> 32);
+    return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
 // min-heap of unique 64-bit keys with stride-32 (interleaved) storage
@@ -170,7 +175,8 @@ __device__ __forceinline__ int warp_argmin(uint64_t v)
 }
 
 struct Decode {
-    int64_t step_end, step_idx, R, ohat;
+    int64_t step_end, R, ohat;
+    int32_t step_idx;        // steps ended; the step budget keeps it and every completion step below 2^31
     int32_t kv_res, kv_rsv;  // resident <= reserved <= C < 2^31 tokens
     uint64_t pend_top, act_top;
     int32_t n_act, q, pend_n, act_n, w_head, w_n;
@@ -216,20 +222,21 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
         // ends is the least of the steps before the next completion, the steps
         // before that term changes, and the steps that end by the limit.
         while (s.stepping && s.step_end <= limit && s.w_n == 0) {
-            const int64_t m_fin = (int64_t)(s.act_top >> kKeyBits) - s.step_idx - 1;  // <= 2^20
+            const int32_t m_fin = (int32_t)(s.act_top >> kKeyBits) - s.step_idx - 1;  // <= 2^20
             if (m_fin <= 0) break;
-            const int64_t n = s.n_act;
+            const int32_t n = s.n_act;
             const int64_t q1 = kv_term(s.kv_res + n, P);  // KV term of the next step
             const int64_t S = P.dec_base + P.dec_seq * n + q1;
             // plain end j happens at step_end + (j - 1) S <= limit (usually the binding bound)
-            int64_t m = m_fin;
+            int32_t m = (int32_t)m_fin;
             const int64_t span = limit - s.step_end;
-            if ((m_fin - 1) * S > span) {  // then span < 2^20 * 2^37
-                m = (span < (int64_t(1) << 56) ? floor_div_small(span, S) : span / S) + 1;
+            if ((int64_t)(m - 1) * S > span) {  // then span < 2^20 * 2^37
+                m = (int32_t)(span < (int64_t(1) << 56) ? floor_div_small(span, S) : span / S) + 1;
             }
             const int64_t room = (q1 + 1) * P.kv_div - 1 - s.kv_res;  // the term stays q1 while j n <= room
-            if (m * n > room) {  // the KV term changes first: m = floor(room / n) >= 1
-                m = n <= kRecipN ? (int64_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n])) : room / n;
+            if ((int64_t)m * n > room) {  // the KV term changes first: m = floor(room / n) >= 1
+                m = n <= kRecipN ? (int32_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n]))
+                                 : (int32_t)(room / n);
             }
             if constexpr (kSnap) {
                 // the poll instant falls before this run or inside it: the occupancy
@@ -238,19 +245,20 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                     if (tsnap < s.step_end) {
                         kv_snap = s.kv_res;
                         tsnap = -1;
-                    } else if (tsnap < s.step_end + (m - 1) * S) {
+                    } else if (tsnap < s.step_end + (int64_t)(m - 1) * S) {
                         const int64_t d = tsnap - s.step_end;  // < (m - 1) S < 2^57
                         const int64_t j = (d < (int64_t(1) << 56) ? floor_div_small(d, S) : d / S) + 1;
-                        kv_snap = s.kv_res + j * n;
+                        kv_snap = s.kv_res + j * (int64_t)n;
                         tsnap = -1;
                     }
                 }
             }
+            const int64_t mn = (int64_t)m * n;
             s.step_idx += m;
-            s.kv_res += (int32_t)(m * n);  // stays within the reservation
-            s.R -= m * n;
+            s.kv_res += (int32_t)mn;  // stays within the reservation
+            s.R -= mn;
             if (s.step_idx + 1 > P.max_steps) return CTR_ETIMEOUT;
-            s.step_end += m * S;
+            s.step_end += (int64_t)m * S;
             if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
         }
         // A KV-ready event while a step runs only matters at the step's end (the
@@ -269,7 +277,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.kv_res += s.n_act;
             s.R -= s.n_act;
             s.stepping = false;
-            while (s.act_n > 0 && (int64_t)(s.act_top >> kKeyBits) == s.step_idx) {
+            while (s.act_n > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
                 const int64_t k = (int64_t)(s.act_top & kKeyMask);
                 heap_pop(act, s.act_n, s.act_top);
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);

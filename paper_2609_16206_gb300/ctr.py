@@ -21,6 +21,7 @@ CTR_OK, CTR_EINVAL, CTR_ECUDA, CTR_EOVERFLOW, CTR_ETIMEOUT = 0, -1, -2, -3, -4
 CTR_MAX_INSTANCES = 32
 CTR_MAX_CONST_SETS = 128
 CTR_MAX_REQUESTS = 1 << 23
+CTR_MAX_STEPS_PER_INSTANCE = (1 << 31) - (1 << 21)
 CTR_SCORE_N_CONST = 13
 CTR_SCORE_MAX_INST = 256
 CTR_WS_SIMULATE = 0

@@ -82,7 +82,7 @@ class SimCfg:
     n_classes: int = 2
     ttft_slo_us: tuple = (1_000_000, 5_000_000)
     tpot_slo_us: tuple = (100_000, 250_000)
-    max_steps_per_instance: int = 1 << 40
+    max_steps_per_instance: int = (1 << 31) - (1 << 21)  # the largest budget the library accepts
     cap_pending: int = 1024
     cap_waiting: int = 1024
     cap_active: int = 1024

@@ -36,7 +36,28 @@ def test_exports_every_declared_function(libctr):
 def test_static_entry_points_run_without_gpu(libctr):
     libctr.ctr_strerror.restype = ctypes.c_char_p
     assert libctr.ctr_strerror(-3).decode().startswith("a fixed-capacity")
-    assert libctr.ctr_abi_version() == 4
+    assert libctr.ctr_abi_version() == 5
+
+
+def test_step_budget_bound_checked_on_the_host():
+    """max_steps_per_instance is accepted up to CTR_MAX_STEPS_PER_INSTANCE (the
+    kernel's step counters are 32-bit) and rejected above it, before any device
+    work (zero rows)."""
+    from paper_2609_16206_gb300 import ctr
+    from paper_2609_16206_gb300 import workloads as W
+    L = ctr.lib()
+    sets = ctr.consts_array([W.CALIBRATED])
+    pols = (ctypes.c_int32 * 1)(0)
+
+    def call(steps):
+        cfg = ctr.sim_cfg_struct(W.SimCfg(max_steps_per_instance=steps))
+        return L.ctr_simulate(ctypes.byref(cfg), sets, 1, pols, 1, ctr.CtrRequests(), 0, 0, None, None, None, None,
+                              None, None, None, 0, None)
+    assert W.SimCfg().max_steps_per_instance == ctr.CTR_MAX_STEPS_PER_INSTANCE == (1 << 31) - (1 << 21)
+    assert call(ctr.CTR_MAX_STEPS_PER_INSTANCE) == ctr.CTR_OK
+    assert call(1) == ctr.CTR_OK
+    assert call(ctr.CTR_MAX_STEPS_PER_INSTANCE + 1) == ctr.CTR_EINVAL
+    assert call(0) == ctr.CTR_EINVAL
 
 
 def test_struct_layout_matches_header(tmp_path):
