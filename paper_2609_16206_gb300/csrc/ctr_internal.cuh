@@ -67,6 +67,9 @@ struct ConstsDev {
     uint64_t poll_recip;  // floor((2^64 - 1) / poll_us)
 };
 
+// The host validates pre_tok, xfer_tok <= 2^20, dec_seq <= 2^16, kv_div <= 2^31
+// and max_steps <= 2^31 - 2^21, so the kernel takes their products with
+// 32-bit counts as single 32 x 32-bit multiplies of the low words.
 struct SimParams {
     int32_t n_pre, n_dec;
     int64_t kv_cap;

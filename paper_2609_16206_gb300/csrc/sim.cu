@@ -226,14 +226,15 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             if (m_fin <= 0) break;
             const int32_t n = s.n_act;
             const int64_t q1 = kv_term(s.kv_res + n, P);  // KV term of the next step
-            const int64_t S = P.dec_base + P.dec_seq * n + q1;
+            const int64_t S = P.dec_base + (int64_t)(int32_t)P.dec_seq * n + q1;
             // plain end j happens at step_end + (j - 1) S <= limit (usually the binding bound)
             int32_t m = (int32_t)m_fin;
             const int64_t span = limit - s.step_end;
             if ((int64_t)(m - 1) * S > span) {  // then span < 2^20 * 2^37
                 m = (int32_t)(span < (int64_t(1) << 56) ? floor_div_small(span, S) : span / S) + 1;
             }
-            const int64_t room = (q1 + 1) * P.kv_div - 1 - s.kv_res;  // the term stays q1 while j n <= room
+            // the term stays q1 while j n <= room; q1 + 1 <= 2^31 and kv_div <= 2^31
+            const int64_t room = (int64_t)((uint64_t)(uint32_t)(q1 + 1) * (uint32_t)P.kv_div) - 1 - s.kv_res;
             if ((int64_t)m * n > room) {  // the KV term changes first: m = floor(room / n) >= 1
                 m = n <= kRecipN ? (int32_t)div_recip((uint64_t)room, (uint64_t)n, __ldg(&kRecipTable.v[n]))
                                  : (int32_t)(room / n);
@@ -257,7 +258,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.step_idx += m;
             s.kv_res += (int32_t)mn;  // stays within the reservation
             s.R -= mn;
-            if (s.step_idx + 1 > P.max_steps) return CTR_ETIMEOUT;
+            if (s.step_idx >= (int32_t)P.max_steps) return CTR_ETIMEOUT;
             s.step_end += (int64_t)m * S;
             if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
         }
@@ -313,8 +314,8 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 admitted += 1;
             }
             if (s.n_act > 0) {
-                if (s.step_idx + 1 > P.max_steps) return CTR_ETIMEOUT;  // steps started on this instance
-                s.step_end = tev + P.dec_base + P.dec_seq * s.n_act + kv_term(s.kv_res, P);
+                if (s.step_idx >= (int32_t)P.max_steps) return CTR_ETIMEOUT;  // steps started on this instance
+                s.step_end = tev + P.dec_base + (int64_t)(int32_t)P.dec_seq * s.n_act + kv_term(s.kv_res, P);
                 if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
                 s.stepping = true;
                 int pos = pos0;
@@ -605,7 +606,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     } else if (is_dec) {
                         if (learned) {
                             const int64_t na = s.n_act;
-                            const int64_t step = P.dec_base + P.dec_seq * na + kv_term(s.kv_res, P);
+                            const int64_t step = P.dec_base + (int64_t)(int32_t)P.dec_seq * s.n_act + kv_term(s.kv_res, P);
                             const uint64_t hi = __umul64hi((uint64_t)s.R, (uint64_t)step);
                             const uint64_t lo = (uint64_t)s.R * (uint64_t)step;
                             int64_t b;
@@ -678,10 +679,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         ring_n += 1;
                         ring_sum_p += pk;
                         if (run_n == 0) {  // an idle instance starts a batch of this request at once
-                            busy = T + P.pre_base + P.pre_tok * pk;
+                            busy = T + P.pre_base + (int64_t)(int32_t)P.pre_tok * (int32_t)pk;
                             run_n = 1;
                             run_p = pk;
-                            ready = busy + P.xfer_tok * pk;
+                            ready = busy + (int64_t)(int32_t)P.xfer_tok * (int32_t)pk;
                             if (ready >= kTimeLimit) err = CTR_EOVERFLOW;
                         } else {  // queued: its KV-ready time is known when its batch starts
                             if (q_batches > 0 && q_tail + pk <= P.pre_batch) {
@@ -695,8 +696,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     }
                 } else if (live && gl == ip) {
                     const int64_t start = busy > T ? busy : T;
-                    const int64_t end = start + P.pre_base + P.pre_tok * pk;
-                    ready = end + P.xfer_tok * pk;
+                    const int64_t end = start + P.pre_base + (int64_t)(int32_t)P.pre_tok * (int32_t)pk;
+                    ready = end + (int64_t)(int32_t)P.xfer_tok * (int32_t)pk;
                     if (ready >= kTimeLimit) {
                         err = CTR_EOVERFLOW;
                     } else if (ring_n == P.cap_ring) {
