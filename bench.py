@@ -490,7 +490,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "50e37c52408b6ed6": {"warp_inst": 156364486550, "dram_bytes": 30.26e9 + 19.91e9},
+    "e0f5e6a2144eeee9": {"warp_inst": 152675214078, "dram_bytes": 30.45e9 + 20.03e9},
 }
 
 SCORE_DRAM_PER_LAUNCH: dict = {

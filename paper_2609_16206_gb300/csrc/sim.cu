@@ -87,14 +87,15 @@ __device__ __forceinline__ uint64_t div_recip(uint64_t num, uint64_t d, uint64_t
     return q;
 }
 
-// floor(x / d) for 0 <= x < 2^56 and 0 < d < 2^37: an fp32 estimate from
-// 32-bit conversions, then exact integer correction (the estimate is within a
-// few units of the quotient whenever the quotient is below 2^20, the only
-// case the simulator asks for; larger quotients fall back to division).
+// floor(x / d) for 0 <= x < 2^56 and 0 < d < 2^37: an fp32 estimate (both
+// operands rounded to fp32, relative error of the quotient a few 2^-24), then
+// exact integer correction (the estimate is within one unit of the quotient
+// whenever the quotient is below 2^20, the only case the simulator asks for;
+// larger quotients fall back to division).
 __device__ __forceinline__ int64_t floor_div_small(int64_t x, int64_t d)
 {
-    const float xf = fmaf(__uint2float_rn((uint32_t)(x >> 24)), 16777216.0f, __uint2float_rn((uint32_t)(x & 0xFFFFFF)));
-    const float df = fmaf(__uint2float_rn((uint32_t)(d >> 24)), 16777216.0f, __uint2float_rn((uint32_t)(d & 0xFFFFFF)));
+    const float xf = __ll2float_rn(x);
+    const float df = __ll2float_rn(d);
     const float qf = __fdividef(xf, df);
     if (!(qf < 1048576.0f)) return x / d;
     int64_t q = (int64_t)__float2int_rz(qf);
@@ -358,24 +359,22 @@ __device__ __forceinline__ bool row_valid(const SimParams& P, int64_t tb, int la
 }
 
 // argmin of 64-bit values within aligned groups of G lanes (ties -> lowest lane),
-// returned as the lane index inside the group
+// returned as the lane index inside the group: a butterfly minimum, then one
+// ballot for the lanes that hold it (every lane of the warp calls it)
 template <int G>
 __device__ __forceinline__ int group_argmin(uint64_t v, int gl)
 {
     if constexpr (G == 32) {
         return warp_argmin(v);
     } else {
-        int idx = gl;
+        uint64_t m = v;  // the group's minimum, then its lowest lane holding it
 #pragma unroll
         for (int off = G / 2; off > 0; off >>= 1) {
-            const uint64_t ov = __shfl_xor_sync(kFull, v, off, G);
-            const int oi = __shfl_xor_sync(kFull, idx, off, G);
-            if (ov < v || (ov == v && oi < idx)) {
-                v = ov;
-                idx = oi;
-            }
+            const uint64_t o = __shfl_xor_sync(kFull, m, off, G);
+            m = o < m ? o : m;
         }
-        return idx;
+        const uint32_t ball = __ballot_sync(kFull, v == m);
+        return __ffs((ball >> ((threadIdx.x & 31) - gl)) & ((1u << G) - 1u)) - 1;
     }
 }
 
