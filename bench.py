@@ -495,7 +495,7 @@ SIM_INST_PER_LAUNCH: dict = {
 
 SCORE_DRAM_PER_LAUNCH: dict = {
     # 2^20 requests x 64 instances, one launch inside the step (profiles/score_kernel_standalone_2p20x64.md)
-    "6e38b5261e3bff8b": {"read": 9.49e6, "write": 0.0},
+    "7b76efe5e7e4728b": {"read": 9.49e6, "write": 0.0},
 }
 
 

@@ -183,7 +183,12 @@ int ctr_gen_trace(const ctr_trace_cfg* cfg /* host */, int32_t n_replicas, int64
  * its fp32 cost; a slo_class >= 4 gives -1 and NaN.  Inputs must be finite and
  * non-negative.  n_req >= 0, 1 <= n_inst <= CTR_SCORE_MAX_INST.  status is an
  * optional device int32 (NULL ok) set to CTR_ETIMEOUT if the shared-memory
- * staging wait of a block ran past its bound (never expected). */
+ * staging wait of a block ran past its bound (never expected).
+ * The kernel is launched as a programmatic dependent launch: it reads nothing
+ * before the preceding work in the stream has completed, and it lets a
+ * following kernel launched the same way be scheduled while it drains (such a
+ * kernel must wait for its grid dependencies before reading this call's
+ * outputs, as kernels launched that way do). */
 int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_t* slo_class, int64_t n_req,
                     const float* q_tokens, const float* n_active, const float* kv_occ, int32_t n_inst,
                     const float* consts /* host */, int32_t* out_argmin, float* out_cost, int32_t* status,

@@ -260,6 +260,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     if (bulk && tid == 0) {
         asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar) : "memory");
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    // launched as a programmatic dependent: nothing the previous kernel in the stream
+    // writes is read before it has completed; the next launch may be scheduled at once
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (bulk && tid == 0) {
         asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(3u * bytes) : "memory");
         asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                          smem_addr(sm.q)),
@@ -499,15 +505,26 @@ cudaError_t launch_score(const ScoreParams& p, cudaStream_t stream)
     int64_t blocks = (p.n + per_block - 1) / per_block;
     const int64_t cap = (int64_t)sms;
     if (blocks > cap) blocks = cap;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     if (vec) {
         err = cudaFuncSetAttribute(score_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (err != cudaSuccess) return err;
-        score_kernel<true><<<(unsigned)blocks, kThreads, smem, stream>>>(p);
+        err = cudaLaunchKernelEx(&cfg, score_kernel<true>, p);
     } else {
         err = cudaFuncSetAttribute(score_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (err != cudaSuccess) return err;
-        score_kernel<false><<<(unsigned)blocks, kThreads, smem, stream>>>(p);
+        err = cudaLaunchKernelEx(&cfg, score_kernel<false>, p);
     }
+    if (err != cudaSuccess) return err;
     return cudaGetLastError();
 }
 
