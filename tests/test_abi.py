@@ -60,6 +60,31 @@ def test_step_budget_bound_checked_on_the_host():
     assert call(0) == ctr.CTR_EINVAL
 
 
+def test_request_count_bound_checked_on_the_host():
+    """CTR_MAX_REQUESTS requests per replica (the 23-bit request index of the
+    packed heap keys) is accepted and one more is rejected, by every entry
+    that takes a request count, before any device work."""
+    from paper_2609_16206_gb300 import ctr
+    from paper_2609_16206_gb300 import workloads as W
+    L = ctr.lib()
+    M = ctr.CTR_MAX_REQUESTS
+    assert M == 1 << 23
+    cfg = ctr.sim_cfg_struct(W.SimCfg())
+    sets = ctr.consts_array([W.CALIBRATED])
+    pols = (ctypes.c_int32 * 1)(0)
+
+    def sim(n_req):  # zero replicas: validation only
+        return L.ctr_simulate(ctypes.byref(cfg), sets, 1, pols, 1, ctr.CtrRequests(), 0, n_req, None, None, None,
+                              None, None, None, None, 0, None)
+
+    def goodput(n_req):
+        return L.ctr_goodput(ctypes.byref(cfg), ctr.CtrRequests(), 0, 4, n_req, None, None, None, None, None)
+    assert sim(M) == ctr.CTR_OK and sim(M + 1) == ctr.CTR_EINVAL and sim(-1) == ctr.CTR_EINVAL
+    assert goodput(M) == ctr.CTR_OK and goodput(M + 1) == ctr.CTR_EINVAL
+    tcfg = ctr.trace_cfg_struct(W.TraceCfg())
+    assert L.ctr_gen_trace(ctypes.byref(tcfg), 1, 0, M + 1, ctr.CtrRequests(), None) == ctr.CTR_EINVAL
+
+
 def test_struct_layout_matches_header(tmp_path):
     from paper_2609_16206_gb300 import ctr
     structs = {"ctr_requests": ctr.CtrRequests, "ctr_trace_cfg": ctr.CtrTraceCfg, "ctr_sim_cfg": ctr.CtrSimCfg,
