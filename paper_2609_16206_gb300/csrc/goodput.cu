@@ -2,10 +2,11 @@
 // the count of requests meeting both SLOs of their class (sec. IV-B targets,
 // Table 2 goodput) and the exact nearest-rank P99 TTFT (Table 2 column).
 //
-// One 256-thread block per row.  Pass 0 reads the row once and reduces the
-// met count and the TTFT range; the P99 is then selected exactly by a radix
-// select over (TTFT - min) with 11-bit digits, most significant first, each
-// pass histogramming the candidates that still match the digits chosen so far
+// One 512-thread block per row (two blocks per SM at 64 registers a
+// thread).  Pass 0 reads the row once and reduces the met count and the TTFT
+// range; the P99 is then selected exactly by a radix select over
+// (TTFT - min) with 11-bit digits, most significant first, each pass
+// histogramming the candidates that still match the digits chosen so far
 // (2048 shared-memory bins).  When the row fits (kStage), pass 0 also keeps
 // its TTFTs in shared memory as 32-bit values and the select passes read them
 // there, so a row crosses HBM once; a row with a TTFT outside [0, 2^32) or too
@@ -15,7 +16,7 @@
 namespace ctr {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 512;
 constexpr int kDigit = 11;
 constexpr int kBins = 1 << kDigit;
 
@@ -40,7 +41,7 @@ __device__ T block_reduce(T v, T identity, Op op, T* scratch)
 }
 
 template <bool kStage>
-__global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P)
+__global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParams P)
 {
     __shared__ uint32_t hist[kBins];
     __shared__ int64_t red64[kThreads / 32];
@@ -53,13 +54,14 @@ __global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P
         const int64_t tb = (row / P.rows_per_replica) * n;
         const int64_t ob = row * n;
         int64_t met = 0, mn = INT64_MAX, mx = INT64_MIN;
-        // 4 elements per thread per round, all loads issued before any is used (the pass is latency-bound)
-        for (int64_t base = tid; base < n; base += (int64_t)kThreads * 4) {
-            int64_t tf[4], td[4], ta[4];
-            int32_t ov[4];
-            uint32_t cv[4];
+        // 2 elements per thread per round, all loads issued before any is used (the pass is latency-bound;
+        // more elements in flight spill at 64 registers and lose more than they hide)
+        for (int64_t base = tid; base < n; base += (int64_t)kThreads * 2) {
+            int64_t tf[2], td[2], ta[2];
+            int32_t ov[2];
+            uint32_t cv[2];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
+            for (int u = 0; u < 2; ++u) {
                 const int64_t k = base + (int64_t)u * kThreads;
                 if (k < n) {
                     tf[u] = __ldg(&P.t_first[ob + k]);
@@ -70,7 +72,7 @@ __global__ void __launch_bounds__(kThreads) goodput_kernel(const GoodputParams P
                 }
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
+            for (int u = 0; u < 2; ++u) {
                 const int64_t k = base + (int64_t)u * kThreads;
                 if (k < n) {
                     const int64_t ttft = tf[u] - ta[u];
