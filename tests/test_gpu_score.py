@@ -183,3 +183,35 @@ def test_random_scoring_problems(orc, seed):
     am, cost = _run(ctr, p, oh, cls, Q, A, kap, consts, offset=int(seed % 2))
     if n:
         _check(orc, p, oh, cls, Q, A, kap, consts, am, cost)
+
+
+def test_chained_launches_read_completed_outputs():
+    """The scorer is launched as a programmatic dependent launch: a call that
+    reads the previous call's output on the same stream (no host sync in
+    between) must see it complete.  Call 1's costs are call 2's prompt
+    lengths; a fill kernel clobbers both output buffers first, so a read that
+    ran ahead of its producer would see NaN or stale values."""
+    ctr = need_gpu()
+    n = 1 << 20
+    p, oh, cls = W.score_requests(n, seed=5)
+    Q, A, kap = W.score_state(64, seed=6)
+    d = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a)).to("cuda", dt)
+    dp, dcls, dQ, dA, dk = d(p, torch.float32), d(cls, torch.uint8), d(Q, torch.float32), d(A, torch.float32), \
+        d(kap, torch.float32)
+    am1 = torch.empty(n, dtype=torch.int32, device="cuda")
+    am2 = torch.empty_like(am1)
+    c1 = torch.empty(n, dtype=torch.float32, device="cuda")
+    c2 = torch.empty_like(c1)
+    for it in range(8):
+        doh = d(oh * (1 + it % 3), torch.float32)
+        c1.fill_(float("nan"))
+        c2.fill_(float("nan"))
+        ctr.ctr_score_batch(dp, doh, dcls, dQ, dA, dk, W.SCORE_CONSTS, am1, c1)
+        ctr.ctr_score_batch(c1, doh, dcls, dQ, dA, dk, W.SCORE_CONSTS, am2, c2)
+        torch.cuda.synchronize()
+        ref_am = torch.empty_like(am2)
+        ref_c = torch.empty_like(c2)
+        ctr.ctr_score_batch(c1.clone(), doh, dcls, dQ, dA, dk, W.SCORE_CONSTS, ref_am, ref_c)
+        torch.cuda.synchronize()
+        assert not torch.isnan(c1).any() and not torch.isnan(c2).any(), it
+        assert torch.equal(am2, ref_am) and torch.equal(c2, ref_c), it
