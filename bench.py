@@ -490,7 +490,7 @@ def run_ours(args, rank, world, local_rank):
 # (the kernel changed since the count was taken) reports null.
 SIM_INST_PER_LAUNCH: dict = {
     # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "e0f5e6a2144eeee9": {"warp_inst": 152675214078, "dram_bytes": 30.45e9 + 20.03e9},
+    "8e8006b0ee8b8922": {"warp_inst": 152140589272, "dram_bytes": 30.43e9 + 20.00e9},
 }
 
 SCORE_DRAM_PER_LAUNCH: dict = {

@@ -98,8 +98,8 @@ __device__ __forceinline__ int64_t floor_div_small(int64_t x, int64_t d)
     const float df = __ll2float_rn(d);
     const float qf = __fdividef(xf, df);
     if (!(qf < 1048576.0f)) return x / d;
-    int64_t q = (int64_t)__float2int_rz(qf);
-    int64_t r = x - q * d;
+    int32_t q = __float2int_rz(qf);  // within one of the quotient, below 2^20
+    int64_t r = x - (int64_t)q * d;
     while (r < 0) {
         --q;
         r += d;
@@ -304,7 +304,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 const uint32_t k = wait[s.w_head * kWarp];
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
-                if (s.kv_rsv + pk + ok > P.kv_cap) break;
+                if ((uint32_t)s.kv_rsv + (uint32_t)(pk + ok) > (uint32_t)P.kv_cap) break;  // < 2^31 + 2^21
                 if (s.act_n == P.cap_act) return CTR_EOVERFLOW;
                 s.w_head = s.w_head + 1 == P.cap_wait ? 0 : s.w_head + 1;
                 s.w_n -= 1;
