@@ -433,18 +433,22 @@ def run_ours(args, rank, world, local_rank):
     issue_peak = n_sm * 4 * sm_max * 1e6 / 1e9   # G warp-instructions / s
     inst = SIM_INST_PER_LAUNCH.get(_source_hash()) if (R, N) == (4096, 20_000) else None
     sim_roof = {"bound": "alu", "unit": "Gwarp-inst/s", "peak": issue_peak,
-                "peak_source": f"{n_sm} SMs x 4 warp-inst/clk x {sm_max:.0f} MHz (max SM clock)",
+                "peak_source": f"{n_sm} SMs x 4 warp-inst/clk x {sm_max:.0f} MHz (max SM clock, "
+                               + ("MEASURED_PEAKS.json)" if "sm_max_mhz" in peaks else "nominal)"),
                 "achieved": None, "frac": None, "traffic": None}
     if inst is not None:
         sim_roof["achieved"] = inst["warp_inst"] / (per_kernel_ms["sim"] / 1e3) / 1e9
         sim_roof["frac"] = sim_roof["achieved"] / issue_peak
         sim_roof["traffic"] = inst.get("dram_bytes")
     hbm = float(peaks.get("hbm_gbs", 6800.0))
+    hbm_source = ("of measured (MEASURED_PEAKS.json hbm_gbs, a STREAM-style copy)" if "hbm_gbs" in peaks
+                  else "of fallback (6.8 TB/s, an earlier GB300 copy measurement)")
     score_bytes = 17 * N_SCORE_REQ + 3 * 4 * N_SCORE_INST
     pairs_per_s = N_SCORE_REQ * N_SCORE_INST / (rot_ms / 1e3)  # graph-batched launches, inputs from HBM
     score_dram = SCORE_DRAM_PER_LAUNCH.get(_source_hash(SCORE_SOURCES))
     score_roof = {"bound": "hbm", "unit": "GB/s", "achieved": score_bytes / (rot_ms / 1e3) / 1e9,
-                  "peak": hbm, "traffic": None if score_dram is None else score_dram["read"] + score_dram["write"],
+                  "peak": hbm, "peak_source": hbm_source,
+                  "traffic": None if score_dram is None else score_dram["read"] + score_dram["write"],
                   "launch_ms": rot_ms, "launch_ms_in_step": per_kernel_ms["score"],
                   "traffic_note": "no counters for this kernel source" if score_dram is None else
                   f"ncu DRAM read {score_dram['read'] / 1e6:.2f} MB, write {score_dram['write'] / 1e6:.2f} MB in "
@@ -454,6 +458,7 @@ def run_ours(args, rank, world, local_rank):
     score_roof["frac"] = score_roof["achieved"] / hbm
     big_bytes = 17 * big_n + 3 * 4 * N_SCORE_INST
     score_roof_big = {"bound": "hbm", "unit": "GB/s", "achieved": big_bytes / (big_ms / 1e3) / 1e9, "peak": hbm,
+                      "peak_source": hbm_source,
                       "traffic": None, "launch_ms": big_ms, "requests": big_n}
     score_roof_big["frac"] = score_roof_big["achieved"] / hbm
     line = {
