@@ -267,9 +267,11 @@ cudaError_t launch_trace(const TraceParams& p, cudaStream_t stream)
     if (err != cudaSuccess) return err;
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
-    const int warps_per_block = 8;
+    // small blocks spread one warp per replica evenly over the SMs (the kernel is
+    // issue-bound, so the SM holding the most warps sets its time)
+    const int warps_per_block = 4;
     int64_t blocks = (p.n_replicas + warps_per_block - 1) / warps_per_block;
-    const int64_t cap = (int64_t)sms * 8;
+    const int64_t cap = (int64_t)sms * 16;
     if (blocks > cap) blocks = cap;
     trace_kernel<<<(unsigned)blocks, warps_per_block * 32, 0, stream>>>(p);
     return cudaGetLastError();
