@@ -86,7 +86,7 @@ struct SimParams {
     int32_t n_sets, n_pols;
     int32_t pols[8];
     int64_t n_req, n_rows;
-    // per-slot workspace: interleaved [entry][lane] arrays
+    // per-slot workspace: three regions, each lane's entries contiguous within a region
     unsigned char* ws;
     uint32_t* next_row;
     int64_t slot_bytes;

@@ -23,8 +23,9 @@
 // per-lane event loops reproduce the global event order exactly (events at
 // an arrival's own time are processed before it is routed).
 //
-// Per-lane structures live in the workspace slot of the warp, interleaved
-// [entry][lane] so that the lanes' heap tops share cache lines: a min-heap of
+// Per-lane structures live in the workspace slot of the warp, each lane's
+// entries contiguous (a heap's levels then share cache lines, and a sift-down
+// reads both children in one access): a min-heap of
 // pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
 // lanes use the same region as their in-flight ring of prefill end times,
 // packed with the prompt length as end << 21 | p), a min-heap of active
@@ -122,47 +123,52 @@ __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
     return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
-// min-heap of unique 64-bit keys with stride-32 (interleaved) storage
+// Entries per lane of a heap region holding up to cap keys: the heap is 1-based
+// (h[1] the root, h[0] unused) and a sift-down reads the children 2i and 2i + 1
+// as one 16-byte word, so the region has cap + 2 entries rounded up to even.
+__host__ __device__ __forceinline__ int64_t heap_stride(int64_t cap) { return (cap + 3) & ~int64_t(1); }
+
+// min-heap of unique 64-bit keys in h[1..n]; each lane's heap is contiguous
 __device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
 {
-    int i = n++;
-    while (i > 0) {
-        const int parent = (i - 1) >> 1;
-        const uint64_t pv = h[parent * kWarp];
+    int i = ++n;
+    while (i > 1) {
+        const int parent = i >> 1;
+        const uint64_t pv = h[parent];
         if (pv < key) break;
-        h[i * kWarp] = pv;
+        h[i] = pv;
         i = parent;
     }
-    h[i * kWarp] = key;
-    if (i == 0) top = key;
+    h[i] = key;
+    if (i == 1) top = key;
 }
 
 __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
 {
-    const int m = --n;
-    if (m == 0) {
+    const int m = n--;  // the last key moves into the hole left at the root
+    if (m == 1) {
         top = kEmpty;
         return;
     }
-    const uint64_t last = h[m * kWarp];
-    int i = 0;
+    const uint64_t last = h[m];
+    const int sz = m - 1;
+    int i = 1;
     for (;;) {
-        int c = 2 * i + 1;
-        if (c >= m) break;
-        uint64_t cv = h[c * kWarp];
-        if (c + 1 < m) {
-            const uint64_t rv = h[(c + 1) * kWarp];
-            if (rv < cv) {
-                cv = rv;
-                ++c;
-            }
+        const int c = 2 * i;
+        if (c > sz) break;
+        const ulonglong2 ch = *reinterpret_cast<const ulonglong2*>(h + c);  // c even: a 16-byte word
+        uint64_t cv = ch.x;
+        int ci = c;
+        if (c < sz && ch.y < cv) {
+            cv = ch.y;
+            ci = c + 1;
         }
         if (last < cv) break;
-        h[i * kWarp] = cv;
-        i = c;
+        h[i] = cv;
+        i = ci;
     }
-    h[i * kWarp] = last;
-    top = h[0];
+    h[i] = last;
+    top = h[1];
 }
 
 // argmin over the lanes of 64-bit values (ties -> lowest lane)
@@ -194,7 +200,7 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
         if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
         int pos = s.w_head + s.w_n;
         if (pos >= P.cap_wait) pos -= P.cap_wait;
-        wait[pos * kWarp] = k;
+        wait[pos] = k;
         s.w_n += 1;
     }
     return CTR_OK;
@@ -301,7 +307,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             const int pos0 = s.w_head;
             int admitted = 0;
             while (s.w_n > 0) {
-                const uint32_t k = wait[s.w_head * kWarp];
+                const uint32_t k = wait[s.w_head];
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
                 if ((uint32_t)s.kv_rsv + (uint32_t)(pk + ok) > (uint32_t)P.kv_cap) break;  // < 2^31 + 2^21
@@ -321,7 +327,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 s.stepping = true;
                 int pos = pos0;
                 for (int i = 0; i < admitted; ++i) {  // first token at the end of this step
-                    const uint32_t k = wait[pos * kWarp];
+                    const uint32_t k = wait[pos];
                     P.t_first[ob + k] = s.step_end;
                     pos = pos + 1 == P.cap_wait ? 0 : pos + 1;
                 }
@@ -407,10 +413,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
     const int64_t slot = (int64_t)blockIdx.x * kWarpsPerBlock + (threadIdx.x >> 5);
     if (slot >= P.n_slots) return;
     unsigned char* sb = P.ws + slot * P.slot_bytes;
-    uint64_t* pend = reinterpret_cast<uint64_t*>(sb) + lane;
-    int64_t* ring = reinterpret_cast<int64_t*>(sb) + lane;
-    uint64_t* act = reinterpret_cast<uint64_t*>(sb + P.off_act) + lane;
-    uint32_t* wait = reinterpret_cast<uint32_t*>(sb + P.off_wait) + lane;
+    const int64_t pr_stride = heap_stride(P.cap_pr);
+    uint64_t* pend = reinterpret_cast<uint64_t*>(sb) + lane * pr_stride;  // decode lanes: 1-based heap
+    int64_t* ring = reinterpret_cast<int64_t*>(sb) + lane * pr_stride;    // prefill lanes: ring from 0
+    uint64_t* act = reinterpret_cast<uint64_t*>(sb + P.off_act) + lane * heap_stride(P.cap_act);
+    uint32_t* wait = reinterpret_cast<uint32_t*>(sb + P.off_wait) + lane * P.cap_wait;
 
     const bool is_pre = gl < P.n_pre;
     const bool is_dec = gl >= P.n_pre && gl < P.n_pre + P.n_dec;
@@ -477,7 +484,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         int pos = ring_head;
                         int64_t pmax = 0;
                         while (run_n < ring_n) {
-                            const int64_t pj = ring[pos * kWarp] & kRingPMask;
+                            const int64_t pj = ring[pos] & kRingPMask;
                             if (run_n > 0 && run_p + pj > P.pre_batch) break;
                             run_p += pj;
                             pmax = pj > pmax ? pj : pmax;
@@ -506,7 +513,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     if (is_dec && live) {
                         int pos = h_i;
                         for (int32_t m = 0; m < m_i; ++m) {
-                            const int64_t v = rings[pos * kWarp + src];
+                            const int64_t v = rings[src * pr_stride + pos];
                             if ((int)((v >> kRingPBits) & 31) == gl - P.n_pre) {
                                 const int64_t ready = e_i + P.xfer_tok * (v & kRingPMask);
                                 if (s.pend_n == P.cap_pend_store) {
@@ -570,7 +577,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                             if constexpr (kSig) ring_sum_p -= ring_front & kRingPMask;
                             ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
                             ring_n -= 1;
-                            ring_front = ring_n > 0 ? ring[ring_head * kWarp] : kNever;
+                            ring_front = ring_n > 0 ? ring[ring_head] : kNever;
                         }
                         if (ring_n == 0) ring_head = 0;
                     }
@@ -674,7 +681,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     } else {
                         int pos = ring_head + ring_n;
                         if (pos >= P.cap_ring) pos -= P.cap_ring;
-                        ring[pos * kWarp] = (k << kRingKShift) | ((int64_t)id << kRingPBits) | pk;
+                        ring[pos] = (k << kRingKShift) | ((int64_t)id << kRingPBits) | pk;
                         ring_n += 1;
                         ring_sum_p += pk;
                         if (run_n == 0) {  // an idle instance starts a batch of this request at once
@@ -706,7 +713,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         int pos = ring_head + ring_n;
                         if (pos >= P.cap_ring) pos -= P.cap_ring;
                         const int64_t e = (end << kRingPBits) | pk;
-                        ring[pos * kWarp] = e;
+                        ring[pos] = e;
                         if (ring_n == 0) ring_front = e;
                         ring_n += 1;
                         if constexpr (kSig) ring_sum_p += pk;
@@ -799,8 +806,8 @@ int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wa
 {
     const int64_t pend_store = (int64_t)cfg.cap_pending + cfg.cap_waiting + 1;  // pending heap entries
     const int64_t pr = pend_store > cfg.cap_prefill_ring ? pend_store : cfg.cap_prefill_ring;
-    const int64_t a = pr * 8 * kWarp;
-    const int64_t b = a + (int64_t)cfg.cap_active * 8 * kWarp;
+    const int64_t a = heap_stride(pr) * 8 * kWarp;
+    const int64_t b = a + heap_stride(cfg.cap_active) * 8 * kWarp;
     const int64_t c = b + (int64_t)cfg.cap_waiting * 4 * kWarp;
     *off_act = a;
     *off_wait = b;
