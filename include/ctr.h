@@ -166,7 +166,11 @@ typedef struct ctr_cost_consts {
  * lognormal laws; the sec. III-C predictor with sec. V-G injected noise;
  * bursty arrivals).  Fills out[r * n_req + k] for replicas
  * g = replica_offset + r, r < n_replicas.  The result is bit-identical to the
- * CPU reference construction (deterministic fp64, integer arrivals).
+ * CPU reference construction: the variates are computed in fp32 (the trace
+ * is defined in fp32, each step correctly rounded in a fixed order, with the
+ * log / exp / normal-quantile functions written out from named methods and
+ * the distribution parameters rounded once from the caller's doubles), and
+ * arrivals are integer prefix sums.
  * n_req 0..CTR_MAX_REQUESTS; n_replicas >= 0; replica_offset >= 0. */
 int ctr_gen_trace(const ctr_trace_cfg* cfg /* host */, int32_t n_replicas, int64_t replica_offset,
                   int64_t n_req, ctr_requests out, void* stream);

@@ -1,8 +1,9 @@
 """Compile libctr.so (the CUDA library behind include/ctr.h) in-tree for sm_103a.
 
 Each translation unit compiles in parallel with nvcc; the trace unit is built
-with -fmad=false so that no fp64 product is fused (its arithmetic must be
-bit-identical to the CPU construction).  Outputs: csrc/../_build/*.o and
+with -fmad=false so that no fp32 product is fused into an add (the trace is
+defined in fp32, each operation rounded on its own, and must be bit-identical
+to the CPU construction, which is compiled with -ffp-contract=off).  Outputs: csrc/../_build/*.o and
 libctr.so next to this file (both git-ignored).
 """
 from __future__ import annotations
