@@ -86,3 +86,47 @@ def test_ablation_mask_bounds(orc):
     tr = orc.gen_trace(wl.trace, 10)
     assert orc.simulate(wl.sim, W.CALIBRATED.replace(ablate=8), 0, tr)["status"] == orc.EINVAL
     assert orc.simulate(wl.sim, W.CALIBRATED, 5, tr)["status"] == orc.EINVAL
+
+
+def test_power_of_two_cheaper_sampled_candidate_wins(orc):
+    """sec. V-D: of the two sampled candidates of a pool, the one with the lower
+    full learned cost is taken (ties to the lower index).  On a 2P+6D row with
+    the proxy's ledger backlog and the pressure feature removed, every cost is
+    re-derived from the row's own outputs (the prefill ledger holds requests
+    whose prefill has not ended at t_k, the decode ledger those not completed),
+    so each choice is checked against the two costs it had to compare."""
+    wl = W.replica_sweep()
+    tr = orc.gen_trace(wl.trace, 2500, replica=6)
+    cc = W.CALIBRATED.replace(proxy_backlog=1, ablate=W.ABLATE_PRESSURE)
+    res = orc.simulate(wl.sim, cc, W.POLICY_LEARNED_P2, tr)
+    assert res["status"] == 0
+    t = tr["arrival_us"].astype(np.int64)
+    p = tr["prompt_len"].astype(np.int64)
+    oh = tr["pred_out"].astype(np.int64)
+    cls = tr["slo_class"].astype(np.int64)
+    ip, idc = res["i_pre"].astype(np.int64), res["i_dec"].astype(np.int64)
+    work_pre = cc.tau_pre0_us + cc.tau_pre_us * p
+    work_dec = oh * cc.tau_dec_us
+    clamp = 1 << 40
+    decided = {"pre": 0, "dec": 0}
+    for k in range(t.size):
+        tk, sig = int(t[k]), int(cc.sigma_q8[cls[k]])
+
+        def cost(pool, i):
+            if pool == "pre":
+                m = (ip[:k] == i) & (res["pre_end_us"][:k] > tk)
+                own, led = int(work_pre[k]), min(clamp, int(work_pre[:k][m].sum()))
+            else:
+                m = (idc[:k] == i) & (res["t_done_us"][:k] > tk)
+                own, led = int(work_dec[k]), min(clamp, int(work_dec[:k][m].sum()))
+            return (cc.w_b_q8 * led + cc.w_s_q8 * own) * sig + cc.w_q_us * int(m.sum()) * 65536
+
+        for pool, n_pool, chosen in (("pre", wl.sim.n_prefill, ip[k]), ("dec", wl.sim.n_decode, idc[k])):
+            pair = sorted(_p2_pair(orc, k, int(t[k]), n_pool, pool))
+            assert len(pair) == 2
+            costs = [cost(pool, i) for i in pair]
+            want = pair[1] if costs[1] < costs[0] else pair[0]
+            assert chosen == want, (k, pool, pair, costs, chosen)
+            decided[pool] += costs[0] != costs[1]
+    # the rule is exercised: most choices are between candidates of different cost
+    assert decided["pre"] > t.size // 2 and decided["dec"] > t.size // 2
