@@ -179,7 +179,10 @@ size_t ctr_workspace_bytes(int32_t which, const ctr_sim_cfg* cfg, int64_t n_rows
     int wpb = 0, blocks = 0;
     const int64_t resident = sim_max_resident_warps(&wpb, &blocks);
     if (resident <= 0) return 0;
-    const int64_t slots = n_rows < resident ? (n_rows > 0 ? n_rows : 1) : resident;
+    // one slot per persistent warp, and a warp carries 32 / width rows
+    const int64_t rows_per_warp = 32 / sim_group_width(cfg->n_prefill + cfg->n_decode);
+    const int64_t warps = (n_rows + rows_per_warp - 1) / rows_per_warp;
+    const int64_t slots = warps < resident ? (warps > 0 ? warps : 1) : resident;
     return (size_t)(256 + slots * slot);
 }
 

@@ -214,7 +214,8 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
 // poll; tsnap <= T), then set tsnap to -1.
 template <bool kSnap>
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
-                                              uint32_t* wait, int64_t tb, int64_t ob, int64_t& tsnap, int64_t& kv_snap)
+                                              uint32_t* wait, int64_t tb, int64_t ob, int64_t& tsnap, int64_t& kv_snap,
+                                              bool track_ohat)
 {
     for (;;) {
         // Plain step ends first: the step ends by T, no request finishes with
@@ -290,12 +291,11 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 heap_pop(act, s.act_n, s.act_top);
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
-                const int64_t ohk = __ldg(&P.trace.pred_out[tb + k]);
                 s.n_act -= 1;
                 s.q -= 1;
                 s.kv_res -= (int32_t)(pk + ok);
                 s.kv_rsv -= (int32_t)(pk + ok);
-                s.ohat -= ohk;
+                if (track_ohat) s.ohat -= __ldg(&P.trace.pred_out[tb + k]);
                 P.t_done[ob + k] = tev;
             }
         }
@@ -435,6 +435,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         const int set = has_row ? (int)((row / P.n_pols) % P.n_sets) : 0;
         const int pol = has_row ? P.pols[row % P.n_pols] : CTR_POLICY_ROUND_ROBIN;
         const ConstsDev& cc = P.sets[set];
+        // the in-flight sum of predicted lengths is read only by the length heuristic and the proxy's ledger
+        const bool track_ohat = kSig || pol == CTR_POLICY_LENGTH_HEURISTIC;
         const int64_t tb = rep * n;
         const int64_t ob = row * n;
 
@@ -570,7 +572,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 last_poll = tp;
                             }
                         }
-                        if (err == CTR_OK) err = decode_advance<kSig>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen);
+                        if (err == CTR_OK) err = decode_advance<kSig>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen, track_ohat);
                     } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
                         while (ring_n > 0 && ring_front <= thr) {
@@ -731,7 +733,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         if (ready >= 0) heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
                         s.q += 1;
                         s.R += ok;
-                        s.ohat += ohk;
+                        if (track_ohat) s.ohat += ohk;
                     }
                 }
                 if (gl == j) my_route = ((uint32_t)ip << 8) | (uint32_t)id;
@@ -754,7 +756,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         }
         if (live && is_dec) {
             int64_t no_snap = -1;
-            err = decode_advance<false>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen);
+            err = decode_advance<false>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, track_ohat);
         }
 
 #pragma unroll
