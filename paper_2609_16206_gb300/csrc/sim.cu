@@ -186,7 +186,7 @@ struct Decode {
     int32_t step_idx;        // steps ended; the step budget keeps it and every completion step below 2^31
     int32_t kv_res, kv_rsv;  // resident <= reserved <= C < 2^31 tokens
     uint64_t pend_top, act_top;
-    int32_t n_act, q, pend_n, act_n, w_head, w_n;
+    int32_t n_act, q, pend_n, w_head, w_n;  // n_act is also the active heap's size
     bool stepping;
 };
 
@@ -286,12 +286,11 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.kv_res += s.n_act;
             s.R -= s.n_act;
             s.stepping = false;
-            while (s.act_n > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
+            while (s.n_act > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
                 const int64_t k = (int64_t)(s.act_top & kKeyMask);
-                heap_pop(act, s.act_n, s.act_top);
+                heap_pop(act, s.n_act, s.act_top);
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
-                s.n_act -= 1;
                 s.q -= 1;
                 s.kv_res -= (int32_t)(pk + ok);
                 s.kv_rsv -= (int32_t)(pk + ok);
@@ -311,13 +310,12 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
                 if ((uint32_t)s.kv_rsv + (uint32_t)(pk + ok) > (uint32_t)P.kv_cap) break;  // < 2^31 + 2^21
-                if (s.act_n == P.cap_act) return CTR_EOVERFLOW;
+                if (s.n_act == P.cap_act) return CTR_EOVERFLOW;
                 s.w_head = s.w_head + 1 == P.cap_wait ? 0 : s.w_head + 1;
                 s.w_n -= 1;
                 s.kv_rsv += (int32_t)(pk + ok);
                 s.kv_res += (int32_t)pk;
-                s.n_act += 1;
-                heap_push(act, s.act_n, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
+                heap_push(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
                 admitted += 1;
             }
             if (s.n_act > 0) {
@@ -453,11 +451,15 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         Decode s;
         s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.R = 0; s.ohat = 0;
         s.pend_top = kEmpty; s.act_top = kEmpty;
-        s.n_act = 0; s.q = 0; s.pend_n = 0; s.act_n = 0; s.w_head = 0; s.w_n = 0;
+        s.n_act = 0; s.q = 0; s.pend_n = 0; s.w_head = 0; s.w_n = 0;
         s.stepping = false;
-        int64_t busy = 0, ring_front = kNever;  // prefill lanes: ring_front = front entry (end << 21 | p)
-        int64_t ring_sum_p = 0;                  // prompt tokens of the prefills in the ring
-        int32_t ring_head = 0, ring_n = 0;
+        // A lane simulates a prefill or a decode instance, never both, so a prefill
+        // lane keeps its state in decode fields it does not use (fewer live registers).
+        int64_t& busy = s.step_end;    // end of the last prefill (of the running batch, when batched)
+        int64_t& ring_front = s.ohat;  // the ring's front entry (end << 21 | p), read while ring_n > 0
+        int64_t& ring_sum_p = s.R;     // prompt tokens of the prefills in the ring
+        int32_t& ring_head = s.w_head;
+        int32_t& ring_n = s.w_n;
         int64_t kv_seen = 0, last_poll = -1;     // decode lanes: occupancy at the last poll instant
         int32_t rr_p = 0, rr_d = 0;
         uint64_t h = 0;
@@ -547,13 +549,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
             uint32_t my_route = 0;
             const int cnt = (int)(n - base < G ? n - base : G);
             for (int j = 0; j < cnt; ++j) {
-                const int64_t k = base + j;
                 const int64_t T = __shfl_sync(kFull, my_t, j, G);
-                const uint32_t pc = __shfl_sync(kFull, my_pc, j, G);
-                const int64_t pk = pc & 0xFFFFFFu;
-                const int ck = (int)(pc >> 24);
-                const int64_t ok = __shfl_sync(kFull, my_o, j, G);
-                const int64_t ohk = __shfl_sync(kFull, my_oh, j, G);
 
                 // 1. advance every instance to the arrival time
                 if constexpr (kBat) {
@@ -587,6 +583,13 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 if (__ballot_sync(kFull, err != CTR_OK) & gmask) live = false;
 
                 __syncwarp();  // the lanes leave their event loops at different passes: regroup
+                // the request's features (read after the advance, which does not need them)
+                const int64_t k = base + j;
+                const uint32_t pc = __shfl_sync(kFull, my_pc, j, G);
+                const int64_t pk = pc & 0xFFFFFFu;
+                const int ck = (int)(pc >> 24);
+                const int64_t ok = __shfl_sync(kFull, my_o, j, G);
+                const int64_t ohk = __shfl_sync(kFull, my_oh, j, G);
                 // 2. price the candidates and take the argmin of each pool
                 uint64_t cost = kEmpty;
                 if (live && pol != CTR_POLICY_ROUND_ROBIN) {
