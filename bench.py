@@ -116,6 +116,56 @@ def oracle_rate(n_replicas: int, n_req: int, cores: int):
     return routed / dt, routed, dt
 
 
+def sampled_parity(wl, offset, R, N, pols, tr, rstat, rhash, met, p99, score_in, score_state, sam, scost):
+    """The benchmarked launch checked against the oracle on sampled rows,
+    outside every timed region (the outputs of the last step: the timed
+    steps and the end-to-end pass compute the same inputs).  The device trace
+    of the first and last three replicas (all three seeds) must equal the
+    oracle's bit for bit, every policy's row status and hash must equal the
+    oracle simulation's, and so must the goodput count and P99 TTFT; 4,096
+    sampled scorer requests must meet the scorer's bar (argmin identical
+    outside the 1e-5 near-tie band, cost within 1e-6 relative)."""
+    import numpy as np
+
+    import oracle
+    t0 = time.perf_counter()
+    reps = sorted({0, 1, 2, R - 3, R - 2, R - 1} & set(range(R)))
+    stat = rstat.cpu().numpy()
+    hsh = rhash.cpu().numpy().astype(np.uint64)
+    met_h, p99_h = met.cpu().numpy(), p99.cpu().numpy()
+    bad, n_rows = [], 0
+    for r in reps:
+        ref = oracle.gen_trace(wl.trace, N, replica=offset + r)
+        for key, v in ref.items():
+            if not np.array_equal(tr[key][r].cpu().numpy(), v):
+                bad.append(f"trace {key} replica {offset + r}")
+        for j, pol in enumerate(pols):
+            row = r * len(pols) + j
+            n_rows += 1
+            o = oracle.simulate(wl.sim, W.CALIBRATED, pol, ref)
+            if int(stat[row]) != o["status"] or (o["status"] == 0 and int(hsh[row]) != o["hash"]):
+                bad.append(f"row {row}")
+            elif o["status"] == 0:
+                if (int(met_h[row]), int(p99_h[row])) != oracle.goodput(wl.sim, ref, o["t_first_us"], o["t_done_us"]):
+                    bad.append(f"goodput row {row}")
+    p, oh, cls = score_in
+    Q, A, kap = score_state
+    idx = np.sort(np.random.default_rng(0).choice(p.size, 4096, replace=False))
+    am, best, second = oracle.score_batch(p[idx], oh[idx], cls[idx], Q, A, kap, W.SCORE_CONSTS)
+    am_d = sam.cpu().numpy()[idx]
+    cost_d = scost.cpu().numpy()[idx].astype(np.float64)
+    strict = (second - best) / best >= 1e-5
+    chosen = oracle.score_pairs(p, oh, cls, idx, am_d, Q, A, kap, W.SCORE_CONSTS)
+    score_ok = bool(np.array_equal(am_d[strict], am[strict]) and np.max(np.abs(cost_d - chosen) / chosen) <= 1e-6
+                    and np.all(chosen <= best * (1 + 1e-5)))
+    if not score_ok:
+        bad.append("scorer")
+    return {"ok": not bad, "rows": n_rows, "replicas": [offset + r for r in reps], "policies": len(pols),
+            "checks": "trace rows bit-exact; row status + hash; goodput met + P99; scorer argmin + cost",
+            "scorer_requests": int(idx.size), "mismatches": bad[:8],
+            "seconds": round(time.perf_counter() - t0, 2)}
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return 0
@@ -421,6 +471,11 @@ def run_ours(args, rank, world, local_rank):
     big_ms = e0.elapsed_time(e1) / reps
     del graph, big
 
+    # ---- parity of the benchmarked launch itself, outside every timed region: the last step's trace,
+    # row statuses and hashes, goodput counts and scorer outputs on sampled rows against the oracle
+    parity = sampled_parity(wl, offset, R, N, pols, tr, rstat, rhash, met, p99, (p, oh, cls), (Q, A, kap), sam, scost) \
+        if rank == 0 and not args.no_parity else None
+
     if rank != 0:
         return 0
     peaks = {}
@@ -431,15 +486,24 @@ def run_ours(args, rank, world, local_rank):
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
     issue_peak = n_sm * 4 * sm_max * 1e6 / 1e9   # G warp-instructions / s
-    inst = SIM_INST_PER_LAUNCH.get(_source_hash()) if (R, N) == (4096, 20_000) else None
+    cnt = SIM_SLICE_COUNTERS.get(_source_hash())
     sim_roof = {"bound": "alu", "unit": "Gwarp-inst/s", "peak": issue_peak,
                 "peak_source": f"{n_sm} SMs x 4 warp-inst/clk x {sm_max:.0f} MHz (max SM clock, "
                                + ("MEASURED_PEAKS.json)" if "sm_max_mhz" in peaks else "nominal)"),
-                "achieved": None, "frac": None, "traffic": None}
-    if inst is not None:
-        sim_roof["achieved"] = inst["warp_inst"] / (per_kernel_ms["sim"] / 1e3) / 1e9
+                "achieved": None, "frac": None, "traffic": None,
+                "inst_per_routed_request": None, "lane_efficiency": None, "dram_bytes_per_routed_request": None}
+    if cnt is not None:
+        # executed warp-instructions scale with routed requests (every row group's instruction stream is
+        # fixed by its inputs), so the slice's count per routed request times this launch's routed requests
+        # is this launch's count; DRAM bytes are scaled the same way (the slice holds fewer warps per SM)
+        routed_launch = rows * N
+        sim_roof["achieved"] = cnt["warp_inst_per_routed"] * routed_launch / (per_kernel_ms["sim"] / 1e3) / 1e9
         sim_roof["frac"] = sim_roof["achieved"] / issue_peak
-        sim_roof["traffic"] = inst.get("dram_bytes")
+        sim_roof["traffic"] = cnt["dram_bytes_per_routed"] * routed_launch
+        sim_roof["inst_per_routed_request"] = cnt["warp_inst_per_routed"]
+        sim_roof["lane_efficiency"] = cnt["thread_inst_per_warp_inst"] / 32
+        sim_roof["dram_bytes_per_routed_request"] = cnt["dram_bytes_per_routed"]
+        sim_roof["counters"] = cnt["slice"]
     hbm = float(peaks.get("hbm_gbs", 6800.0))
     hbm_source = ("of measured (MEASURED_PEAKS.json hbm_gbs, a STREAM-style copy)" if "hbm_gbs" in peaks
                   else "of fallback (6.8 TB/s, an earlier GB300 copy measurement)")
@@ -477,11 +541,14 @@ def run_ours(args, rank, world, local_rank):
         "roofline_score": score_roof,
         "roofline_score_2p24": score_roof_big,
         "cpu_baseline": cpu_base,
+        "parity_sampled": parity,
         "e2e": {"value": e2e_value, "unit": "routed requests/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "note": "per step: trace + scorer inputs copied in from pinned host memory (the next step's copy "
                          "overlaps this step's compute on a second stream, double-buffered), simulate + goodput + "
-                         "score, per-row results and scorer outputs copied out",
+                         "score, per-row results and scorer outputs copied out; the host copy of the trace takes "
+                         "the place of on-device trace generation (ctr_gen_trace), so this step does that much "
+                         "less device work than the device-timed step",
                  "steps": e2e_steps},
         "gpu_launches": 5 * args.steps,  # gen, sim, checksum pass, goodput, score
         "clocks": clk,
@@ -490,16 +557,22 @@ def run_ours(args, rank, world, local_rank):
     return 0
 
 
-# Executed warp instructions of one sim_kernel launch on the benchmarked
-# workload (ncu sm__inst_executed.sum), keyed by a hash of csrc/: a stale entry
-# (the kernel changed since the count was taken) reports null.
-SIM_INST_PER_LAUNCH: dict = {
-    # 4,096 replicas x 20,000 requests x 4 policies, one launch (profiles/sim_kernel_replica_sweep_4096x20000.md)
-    "8e8006b0ee8b8922": {"warp_inst": 152140589272, "dram_bytes": 30.43e9 + 20.00e9},
+# Counters of one sim_kernel launch on a slice of the benchmarked workload
+# (ncu sm__inst_executed.sum, smsp__thread_inst_executed.sum and DRAM bytes of
+# 1,024 replicas x 20,000 requests x 4 policies, a few GB on the device),
+# per routed request, keyed by a hash of the simulator's code: a stale entry
+# (the kernel changed since the counters were taken) reports null.
+SIM_SLICE_COUNTERS: dict = {
+    "5e60eff741639c91": {"warp_inst_per_routed": 34340675617 / 81_920_000,
+                         "thread_inst_per_warp_inst": 285008436021 / 34340675617,
+                         "dram_bytes_per_routed": (2.39e9 + 1.57e9) / 81_920_000,
+                         "slice": "ncu on one launch of 1,024 replicas x 20,000 requests x 4 policies "
+                                  "(81.92 M routed requests): 3.434e10 warp-instructions, 2.850e11 thread-"
+                                  "instructions, 2.39 GB DRAM read + 1.57 GB written"},
 }
 
+# DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.
 SCORE_DRAM_PER_LAUNCH: dict = {
-    # 2^20 requests x 64 instances, one launch inside the step (profiles/score_kernel_standalone_2p20x64.md)
     "7b76efe5e7e4728b": {"read": 9.49e6, "write": 0.0},
 }
 
@@ -616,6 +689,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end pass")
+    ap.add_argument("--no-parity", action="store_true", help="skip the sampled oracle check of the benchmarked launch")
     ap.add_argument("--replicas", type=int, default=None,
                     help="replicas per GPU (profiling a smaller case; default: the benchmarked 4,096)")
     ap.add_argument("--requests", type=int, default=None, help="requests per replica (default 20,000)")
