@@ -26,7 +26,9 @@ int cuda_status(cudaError_t e) { return e == cudaSuccess ? CTR_OK : CTR_ECUDA; }
 bool valid_sim_cfg(const ctr_sim_cfg* c)
 {
     if (!c) return false;
-    if (c->n_prefill < 1 || c->n_decode < 1 || c->n_prefill + c->n_decode > CTR_MAX_INSTANCES) return false;
+    if (c->n_prefill < 1 || c->n_decode < 1 || c->n_prefill > CTR_MAX_INSTANCES || c->n_decode > CTR_MAX_INSTANCES)
+        return false;
+    if (c->n_prefill + c->n_decode > CTR_MAX_INSTANCES) return false;  // no overflow: each is <= 32
     if (!in_range(c->kv_cap_tokens, 1, 2147483647LL)) return false;
     if (!in_range(c->pre_base_us, 1, 1LL << 30) || !in_range(c->pre_us_per_tok, 0, 1LL << 20)) return false;
     if (!in_range(c->xfer_us_per_tok, 0, 1LL << 20)) return false;
@@ -105,7 +107,7 @@ int ctr_gen_trace(const ctr_trace_cfg* cfg, int32_t n_replicas, int64_t replica_
         if (cfg->class_thr[i] > (1ull << 32)) return CTR_EINVAL;
         if (i > 0 && cfg->class_thr[i] < cfg->class_thr[i - 1]) return CTR_EINVAL;
     }
-    if (replica_offset + (int64_t)n_replicas > (1LL << 40)) return CTR_EINVAL;
+    if (replica_offset > (1LL << 40) - (int64_t)n_replicas) return CTR_EINVAL;  // offset + count <= 2^40
 
     TraceParams p;
     std::memset(&p, 0, sizeof(p));

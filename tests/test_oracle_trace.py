@@ -118,3 +118,87 @@ def test_replica_seeding_rule(orc):
     assert not np.array_equal(r0["prompt_len"], r3["prompt_len"])
     again = orc.gen_trace(tc, 300, replica=0)
     assert all(np.array_equal(r0[k], again[k]) for k in r0)
+
+
+def test_mmpp_starts_in_the_low_state(orc):
+    """The two-state MMPP starts in its first (low-rate) state: over many
+    replicas the arrivals in the first second average about 3 (the first
+    dwell, mean 10 s, rarely ends that early: e^-0.1 of replicas are still in
+    it at 1 s), not 12; listing the rates the other way round flips it.  The
+    mean rate and the dispersion test above cannot tell which state comes
+    first."""
+    tc = W.replica_sweep().trace
+    n_rep = 2000
+
+    def first_second_mean(cfg):
+        counts = [int(np.sum(orc.gen_trace(cfg, 40, replica=g)["arrival_us"] < 1_000_000)) for g in range(n_rep)]
+        return float(np.mean(counts))
+
+    # exact expectation: rate lam0 until the first switch (exponential, mean 10 s), then lam1
+    # E[count in [0, 1 s)] = lam1 * 1 + (lam0 - lam1) * E[min(D, 1)], E[min(D, 1)] = 10 (1 - e^-0.1)
+    e_min = 10.0 * (1.0 - np.exp(-0.1))
+    low_first = 12.0 + (3.0 - 12.0) * e_min
+    high_first = 3.0 + (12.0 - 3.0) * e_min
+    se = np.sqrt(12.0 / n_rep)
+    a = first_second_mean(tc)
+    b = first_second_mean(tc.replace(rate_mreq=(tc.rate_mreq[1], tc.rate_mreq[0])))
+    assert abs(a - low_first) < 5 * se, (a, low_first)
+    assert abs(b - high_first) < 5 * se, (b, high_first)
+
+
+def test_counter_layout_of_each_request(orc):
+    """The trace spec's counter layout, checked against the KAT-pinned
+    Philox4x32-10 and the separately pinned fp32 functions: replica g uses key
+    seed + (g mod n_seeds) and sub-stream g / n_seeds; request k draws counter
+    (k, sub, 0, 0) for (prompt, mixture, output, noise) and (k, sub, 0, 1) for
+    (class, gap); MMPP dwell j draws (j, sub, 1, 0).  Every field of a few
+    requests of several replicas is rebuilt here from those words."""
+    tc = W.TraceCfg(seed=11, n_seeds=3, arrival_kind=0, rate_mreq=(4000, 4000))
+    f32 = np.float32
+
+    def round_clip(v, lo, hi):
+        y = f32(v) + f32(0.5)
+        if not (y < f32(hi)):
+            return hi
+        return max(lo, int(y))
+
+    for g in (0, 1, 2, 4, 7):
+        tr = orc.gen_trace(tc, 40, replica=g)
+        seed = tc.seed + g % tc.n_seeds
+        key = [seed & 0xFFFFFFFF, seed >> 32]
+        sub = g // tc.n_seeds
+        lam = 0
+        for k in range(40):
+            x = orc.philox4x32_10([k, sub, 0, 0], key)
+            y = orc.philox4x32_10([k, sub, 0, 1], key)
+            zp = orc.det_ndtrif(np.array([x[0]], np.uint32))[0]
+            p = round_clip(orc.det_expf(np.array([f32(tc.prompt_mu) + f32(tc.prompt_sigma) * zp], f32))[0],
+                           tc.prompt_min, tc.prompt_max)
+            short = int(x[1]) < tc.mix_short_thr
+            mu, sg = (tc.short_mu, tc.short_sigma) if short else (tc.long_mu, tc.long_sigma)
+            zo = orc.det_ndtrif(np.array([x[2]], np.uint32))[0]
+            o = round_clip(orc.det_expf(np.array([f32(mu) + f32(sg) * zo], f32))[0], tc.out_min, tc.out_max)
+            zn = orc.det_ndtrif(np.array([x[3]], np.uint32))[0]
+            fac = orc.det_expf(np.array([f32(tc.noise_sigma) * zn], f32))[0]
+            oh = round_clip(f32(o) * fac, tc.pred_min, tc.pred_max)
+            c = int(int(y[0]) >= tc.class_thr[0])
+            lg = orc.det_logf(orc.unit_uniform(np.array([y[1]], np.uint32)))[0]
+            lam += int(f32(-lg) * f32(1e9))
+            assert (int(tr["prompt_len"][k]), int(tr["true_out"][k]), int(tr["pred_out"][k]),
+                    int(tr["slo_class"][k])) == (p, o, oh, c), (g, k)
+            assert int(tr["arrival_us"][k]) == lam // tc.rate_mreq[0], (g, k)
+
+    # MMPP: the first dwell comes from counter (0, sub, 1, 0) of the replica's key
+    mm = W.TraceCfg(seed=5, arrival_kind=1, rate_mreq=(3000, 12000), dwell_mean_us=10_000_000)
+    tr = orc.gen_trace(mm, 400, replica=0)
+    w = orc.philox4x32_10([0, 0, 1, 0], [5, 0])
+    d0 = int(f32(-orc.det_logf(orc.unit_uniform(np.array([w[0]], np.uint32)))[0]) * f32(mm.dwell_mean_us))
+    # arrivals before the first switch follow the low rate exactly
+    lam = 0
+    for k in range(400):
+        y = orc.philox4x32_10([k, 0, 0, 1], [5, 0])
+        lam += int(f32(-orc.det_logf(orc.unit_uniform(np.array([y[1]], np.uint32)))[0]) * f32(1e9))
+        if lam >= 3000 * d0:
+            break
+        assert int(tr["arrival_us"][k]) == lam // 3000, k
+    assert k > 0
