@@ -198,6 +198,16 @@ int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_
                     const float* consts /* host */, int32_t* out_argmin, float* out_cost, int32_t* status,
                     void* stream);
 
+/* ctr_score_stream_probe -- a measurement aid, not a step of the method (the
+ * paper has no counterpart): the memory traffic of ctr_score_batch without its
+ * arithmetic, on the same grid with the same loads and stores, writing
+ * out_argmin[r] = slo_class[r] and out_cost[r] = prompt_len[r] + pred_out[r].
+ * Timed beside the scorer it gives the HBM throughput a kernel of this shape
+ * reaches at that size.  n_req a multiple of 4; float arrays 16-byte aligned,
+ * slo_class 4-byte aligned (CTR_EINVAL otherwise). */
+int ctr_score_stream_probe(const float* prompt_len, const float* pred_out, const uint8_t* slo_class, int64_t n_req,
+                           int32_t* out_argmin, float* out_cost, void* stream);
+
 /* ctr_workspace_bytes -- device workspace ctr_simulate needs to run its
  * widest grid for these sizes on the current device (0 on bad arguments).
  * A smaller workspace is accepted and runs fewer concurrent rows. */

@@ -171,6 +171,25 @@ int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_
     return cuda_status(launch_score(p, (cudaStream_t)stream));
 }
 
+int ctr_score_stream_probe(const float* prompt_len, const float* pred_out, const uint8_t* slo_class, int64_t n_req,
+                           int32_t* out_argmin, float* out_cost, void* stream)
+{
+    if (n_req < 0 || n_req % 4 != 0) return CTR_EINVAL;
+    if (n_req > 0 && (!prompt_len || !pred_out || !slo_class || !out_argmin || !out_cost)) return CTR_EINVAL;
+    if ((((uintptr_t)prompt_len | (uintptr_t)pred_out | (uintptr_t)out_argmin | (uintptr_t)out_cost) % 16u) != 0 ||
+        (uintptr_t)slo_class % 4u != 0)
+        return CTR_EINVAL;
+    ScoreParams p;
+    std::memset(&p, 0, sizeof(p));
+    p.p = prompt_len;
+    p.oh = pred_out;
+    p.cls = slo_class;
+    p.n = n_req;
+    p.argmin = out_argmin;
+    p.cost = out_cost;
+    return cuda_status(launch_stream_probe(p, (cudaStream_t)stream));
+}
+
 size_t ctr_workspace_bytes(int32_t which, const ctr_sim_cfg* cfg, int64_t n_rows, int64_t n_req)
 {
     (void)n_req;

@@ -136,5 +136,6 @@ struct ScoreParams {
     int32_t* status;
 };
 cudaError_t launch_score(const ScoreParams& p, cudaStream_t stream);
+cudaError_t launch_stream_probe(const ScoreParams& p, cudaStream_t stream);  // scorer's traffic only
 
 }  // namespace ctr

@@ -140,20 +140,27 @@ __device__ __forceinline__ bool line_less(float a, float m, int i, float b, floa
     return a < b || (a == b && (m < n || (m == n && i < j)));
 }
 
-// lexicographic (x, m, i) minimum over the warp; every lane gets the result
-__device__ __forceinline__ void warp_min_xmi(float& x, float& m, int& i)
+// An order-preserving 32-bit key of a float: (key(a) < key(b)) == (a < b) for
+// non-NaN a, b (negative values have every bit flipped, others the sign bit set).
+__device__ __forceinline__ uint32_t fkey(float x)
 {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-        const float px = __shfl_xor_sync(0xffffffffu, x, off);
-        const float pm = __shfl_xor_sync(0xffffffffu, m, off);
-        const int pi = __shfl_xor_sync(0xffffffffu, i, off);
-        if (line_less(px, pm, pi, x, m, i)) {
-            x = px;
-            m = pm;
-            i = pi;
-        }
-    }
+    const uint32_t b = __float_as_uint(x);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Lexicographic (x, m, j) minimum over the warp of each lane's candidate,
+// returned to every lane as the winning index j (-1 when no lane has one):
+// three redux.sync minimum reductions, on the key of x, then on the key of m
+// among the lanes holding that x, then on j among those holding both.
+__device__ __forceinline__ int warp_lexmin(bool has, float x, float m, int j)
+{
+    const uint32_t kx = has ? fkey(x) : 0xffffffffu;
+    const uint32_t mx = __reduce_min_sync(0xffffffffu, kx);
+    const bool at_x = has && kx == mx;
+    const uint32_t km = at_x ? fkey(m) : 0xffffffffu;
+    const uint32_t mm = __reduce_min_sync(0xffffffffu, km);
+    const uint32_t kj = at_x && km == mm ? (uint32_t)j : 0xffffffffu;
+    return (int)__reduce_min_sync(0xffffffffu, kj);
 }
 
 // Lower envelope of one class's lines over o_hat >= 0 with one warp, for up to
@@ -162,14 +169,15 @@ __device__ __forceinline__ void warp_min_xmi(float& x, float& m, int& i)
 // among the lines of smaller slope, the one whose crossing with it comes first
 // (ties: smaller slope, then lower index), and the crossing is that segment's
 // left end.  Each step lowers the slope, so the loop ends within n_inst steps,
-// one warp argmin each (a handful for the states seen in practice: the
-// envelope of n random lines has O(log n) segments).  Left ends are kept
-// non-decreasing against rounding.  Segment t stays in lane t % 32, slot
-// t / 32, until the warp writes the segment arrays and the padded breakpoints.
+// one warp minimum each (a handful for the states seen in practice: the
+// envelope of n random lines has O(log n) segments).  A lane's two lines are
+// compared first, then the warp takes the minimum with two redux.sync
+// reductions and a ballot.  Left ends are kept non-decreasing against
+// rounding.  Segment t stays in lane t % 32, slot t / 32, until the warp writes
+// the segment arrays and the padded breakpoints.
 __device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst, int lane)
 {
     const float inf = __int_as_float(0x7f800000);
-    constexpr int kNone = 1 << 20;
     const float sig = P.c[9 + s];
     const float ks = sig * P.c[1] * P.c[6] * P.c[3];
     float a[2], m[2];
@@ -183,41 +191,42 @@ __device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst,
         // a non-finite line (outside the input contract) takes no part, which keeps
         // every comparison below a total order and the warp's decisions uniform
         live[r] = fabsf(a[r]) < inf && fabsf(m[r]) < inf;
-        if (!live[r]) a[r] = m[r] = inf;
     }
-    float ca = a[0], cm = m[0];
-    int ci = live[0] ? lane : kNone;
-    if (live[1] && line_less(a[1], m[1], lane + 32, ca, cm, ci)) {
-        ca = a[1];
-        cm = m[1];
-        ci = lane + 32;
-    }
-    warp_min_xmi(ca, cm, ci);
-    if (ci == kNone) ci = 0;  // no finite line at all (outside the input contract)
+    // the lane's least line, then the warp's: (intercept, slope, index)
+    int r0 = live[0] ? 0 : 1;
+    if (live[0] && live[1] && line_less(a[1], m[1], lane + 32, a[0], m[0], lane)) r0 = 1;
+    int ci = warp_lexmin(live[0] || live[1], r0 ? a[1] : a[0], r0 ? m[1] : m[0], lane + 32 * r0);
+    bool more = ci >= 0;
+    if (!more) ci = 0;  // no finite line at all (outside the input contract): line 0
+    float ca = __shfl_sync(0xffffffffu, ci >= 32 ? a[1] : a[0], ci & 31);
+    float cm = __shfl_sync(0xffffffffu, ci >= 32 ? m[1] : m[0], ci & 31);
     float lo0 = 0.0f, lo1 = 0.0f;
     int id0 = ci, id1 = 0;
     float x_cur = 0.0f;
     int nseg = 1;
-    while (nseg < n_inst) {
+    while (more && nseg < n_inst) {
+        // the lane's first crossing among its lines of smaller slope (x, slope, index)
+        bool has = false;
         float bx = inf, bm = inf;
-        int bi = kNone;
+        int br = 0;
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
-            const int j = lane + 32 * r;
             if (live[r] && m[r] < cm) {
                 const float x = (a[r] - ca) / (cm - m[r]);
-                if (x == x && line_less(x, m[r], j, bx, bm, bi)) {
+                if (x == x && (!has || x < bx || (x == bx && m[r] < bm))) {  // slot 0 (lower index) on full ties
+                    has = true;
                     bx = x;
                     bm = m[r];
-                    bi = j;
+                    br = r;
                 }
             }
         }
-        warp_min_xmi(bx, bm, bi);
-        if (bi == kNone) break;  // warp-uniform: no line of smaller slope is left
-        ca = __shfl_sync(0xffffffffu, bi < 32 ? a[0] : a[1], bi & 31);
-        cm = bm;
-        x_cur = fmaxf(bx, x_cur);
+        const int bi = warp_lexmin(has, bx, bm, lane + 32 * br);  // the warp's first crossing
+        if (bi < 0) break;  // warp-uniform: no line of smaller slope is left
+        const int wl = bi & 31;
+        ca = __shfl_sync(0xffffffffu, bi >= 32 ? a[1] : a[0], wl);
+        cm = __shfl_sync(0xffffffffu, bm, wl);
+        x_cur = fmaxf(__shfl_sync(0xffffffffu, bx, wl), x_cur);
         if (lane == (nseg & 31)) {
             if (nseg < 32) {
                 lo0 = x_cur;
@@ -488,6 +497,61 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     }
 }
 
+// The scorer's memory traffic without its arithmetic or prologue: the same
+// grid, launch attributes, 128-bit streaming loads two vectors ahead and
+// streaming stores, writing class and p + o_hat.  It measures the HBM ceiling
+// the scorer can reach at a given size.
+__global__ void __launch_bounds__(kThreads, 1) stream_probe_kernel(const ScoreParams P)
+{
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int64_t nv = P.n >> 2;
+    const int64_t stride = (int64_t)gridDim.x * kThreads;
+    const float4* p4 = reinterpret_cast<const float4*>(P.p);
+    const float4* o4 = reinterpret_cast<const float4*>(P.oh);
+    const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
+    int4* a4 = reinterpret_cast<int4*>(P.argmin);
+    float4* f4 = reinterpret_cast<float4*>(P.cost);
+    int64_t v = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+    bool has = v < nv;
+    float4 pv = make_float4(0.f, 0.f, 0.f, 0.f), ov = pv, pn = pv, on = pv;
+    uint32_t cv = 0, cn = 0;
+    if (has) {
+        pv = ld_stream(p4 + v);
+        ov = ld_stream(o4 + v);
+        cv = ld_stream_u32(c4 + v);
+    }
+    bool hn = v + stride < nv;
+    if (hn) {
+        pn = ld_stream(p4 + v + stride);
+        on = ld_stream(o4 + v + stride);
+        cn = ld_stream_u32(c4 + v + stride);
+    }
+    while (has) {
+        const int64_t vf = v + 2 * stride;
+        const bool hf = vf < nv;
+        float4 pf = make_float4(0.f, 0.f, 0.f, 0.f), of = pf;
+        uint32_t cf = 0;
+        if (hf) {
+            pf = ld_stream(p4 + vf);
+            of = ld_stream(o4 + vf);
+            cf = ld_stream_u32(c4 + vf);
+        }
+        __stcs(a4 + v, make_int4((int)(cv & 0xFFu), (int)((cv >> 8) & 0xFFu), (int)((cv >> 16) & 0xFFu),
+                                 (int)(cv >> 24)));
+        __stcs(f4 + v, make_float4(pv.x + ov.x, pv.y + ov.y, pv.z + ov.z, pv.w + ov.w));
+        v += stride;
+        has = hn;
+        pv = pn;
+        ov = on;
+        cv = cn;
+        hn = hf;
+        pn = pf;
+        on = of;
+        cn = cf;
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_score(const ScoreParams& p, cudaStream_t stream)
@@ -524,6 +588,30 @@ cudaError_t launch_score(const ScoreParams& p, cudaStream_t stream)
         if (err != cudaSuccess) return err;
         err = cudaLaunchKernelEx(&cfg, score_kernel<false>, p);
     }
+    if (err != cudaSuccess) return err;
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stream_probe(const ScoreParams& p, cudaStream_t stream)
+{
+    if (p.n < 4) return cudaSuccess;
+    int dev = 0, sms = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    int64_t blocks = ((p.n >> 2) + kThreads - 1) / kThreads;
+    if (blocks > sms) blocks = sms;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)blocks);
+    cfg.blockDim = dim3(kThreads);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    err = cudaLaunchKernelEx(&cfg, stream_probe_kernel, p);
     if (err != cudaSuccess) return err;
     return cudaGetLastError();
 }

@@ -89,6 +89,8 @@ def lib():
             L.ctr_gen_trace.restype = C.c_int
             L.ctr_score_batch.argtypes = [vp, vp, vp, i64, vp, vp, vp, i32, C.POINTER(C.c_float), vp, vp, vp, vp]
             L.ctr_score_batch.restype = C.c_int
+            L.ctr_score_stream_probe.argtypes = [vp, vp, vp, i64, vp, vp, vp]
+            L.ctr_score_stream_probe.restype = C.c_int
             L.ctr_workspace_bytes.argtypes = [i32, C.POINTER(CtrSimCfg), i64, i64]
             L.ctr_workspace_bytes.restype = C.c_size_t
             L.ctr_simulate.argtypes = [C.POINTER(CtrSimCfg), C.POINTER(CtrCostConsts), i32, C.POINTER(i32), i32,
@@ -227,6 +229,13 @@ def ctr_score_batch(prompt_len, pred_out, slo_class, q_tokens, n_active, kv_occ,
     _check("ctr_score_batch", lib().ctr_score_batch(
         _ptr(prompt_len), _ptr(pred_out), _ptr(slo_class), int(prompt_len.numel()), _ptr(q_tokens), _ptr(n_active),
         _ptr(kv_occ), int(q_tokens.numel()), cv, _ptr(out_argmin), _ptr(out_cost), _ptr(status), _stream(stream)))
+
+
+def ctr_score_stream_probe(prompt_len, pred_out, slo_class, out_argmin, out_cost, stream=None):
+    """The scorer's memory traffic alone (a measurement aid; see include/ctr.h)."""
+    _check("ctr_score_stream_probe", lib().ctr_score_stream_probe(
+        _ptr(prompt_len), _ptr(pred_out), _ptr(slo_class), int(prompt_len.numel()), _ptr(out_argmin),
+        _ptr(out_cost), _stream(stream)))
 
 
 def ctr_workspace_bytes(which: int, sim_cfg, n_rows: int, n_req: int) -> int:
