@@ -232,6 +232,33 @@ def _source_hash(sources=SIM_SOURCES) -> str:
     return h.hexdigest()[:16]
 
 
+def graph_ms(issue, stream, cap, reps):
+    """Milliseconds per replay of a CUDA graph of the launches `issue(stream)`
+    makes (captured on `cap`, replayed on `stream` after warm-up)."""
+    import torch
+    with torch.cuda.stream(stream):
+        issue(stream)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    cap.wait_stream(stream)
+    with torch.cuda.graph(graph, stream=cap):
+        issue(cap)
+    stream.wait_stream(cap)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            graph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    del graph
+    return e0.elapsed_time(e1) / reps
+
+
 def run_ours(args, rank, world, local_rank):
     import numpy as np
     import torch
@@ -276,7 +303,7 @@ def run_ours(args, rank, world, local_rank):
     sam = torch.empty(N_SCORE_REQ, dtype=torch.int32, device=dev)
     scost = torch.empty(N_SCORE_REQ, dtype=torch.float32, device=dev)
 
-    ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(2)] for k in ("gen", "sim", "goodput", "score")}
+    ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(2)] for k in ("gen", "sim", "score")}
     times = {k: 0.0 for k in ev}
 
     def step(timed: bool):
@@ -286,12 +313,10 @@ def run_ours(args, rank, world, local_rank):
         mark("gen", 0)
         ctr.ctr_gen_trace(wl.trace, R, offset, N, tr, stream=stream)
         mark("gen", 1)
-        mark("sim", 0)
-        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, tr, R, N, tf, td, rhash, rstat, ws, stream=stream)
+        mark("sim", 0)  # simulation, then each row's checksum and goodput in one pass over the outputs
+        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, tr, R, N, tf, td, rhash, rstat, ws, met_count=met,
+                         p99_ttft_us=p99, stream=stream)
         mark("sim", 1)
-        mark("goodput", 0)
-        ctr.ctr_goodput(wl.sim, tr, R, len(pols), N, tf, td, met, p99, stream=stream)
-        mark("goodput", 1)
         mark("score", 0)
         ctr.ctr_score_batch(sp, soh, scls, sQ, sA, skap, W.SCORE_CONSTS, sam, scost, stream=stream)
         mark("score", 1)
@@ -373,8 +398,8 @@ def run_ours(args, rank, world, local_rank):
         b = i % 2
         stream.wait_event(ready[b])
         t_, (p_, oh_, cls_) = bufs[b]
-        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, t_, R, N, tf, td, rhash, rstat, ws, stream=stream)
-        ctr.ctr_goodput(wl.sim, t_, R, len(pols), N, tf, td, met, p99, stream=stream)
+        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, t_, R, N, tf, td, rhash, rstat, ws, met_count=met,
+                         p99_ttft_us=p99, stream=stream)
         ctr.ctr_score_batch(p_, oh_, cls_, sQ, sA, skap, W.SCORE_CONSTS, sam, scost, stream=stream)
         freed[b].record(stream)
         with torch.cuda.stream(stream):
@@ -438,7 +463,12 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     rot_ms = g0.elapsed_time(g1) / (g_reps * rot_sets)
     rot_ok = all(torch.equal(b[3], rot[0][3]) for b in rot[1:])
-    del graph, rot
+    del graph
+    # the same harness around the scorer's traffic alone (ctr_score_stream_probe: its loads and stores on the
+    # same grid, no arithmetic): the HBM throughput a kernel of this shape reaches at this size
+    probe_ms = graph_ms(lambda st: [ctr.ctr_score_stream_probe(b[0], b[1], b[2], b[3], b[4], stream=st) for b in rot],
+                        stream, cap, g_reps) / rot_sets
+    del rot
 
     # ---- the scorer once more on 2^24 requests (285 MB per launch, beyond L2): its HBM roofline
     big_n = 1 << 24
@@ -469,7 +499,10 @@ def run_ours(args, rank, world, local_rank):
     e1.record(stream)
     torch.cuda.synchronize()
     big_ms = e0.elapsed_time(e1) / reps
-    del graph, big
+    del graph
+    big_probe_ms = graph_ms(lambda st: [ctr.ctr_score_stream_probe(b[0], b[1], b[2], b[3], b[4], stream=st)
+                                        for b in (big[i % 2] for i in range(reps))], stream, cap, 1) / reps
+    del big
 
     # ---- parity of the benchmarked launch itself, outside every timed region: the last step's trace,
     # row statuses and hashes, goodput counts and scorer outputs on sampled rows against the oracle
@@ -520,11 +553,19 @@ def run_ours(args, rank, world, local_rank):
                   "timing": f"{rot_sets} buffer sets ({rot_sets * score_bytes / 1e6:.0f} MB, > 4x L2) back to back "
                             f"from one CUDA graph, x{g_reps}; outputs identical across sets: {rot_ok}"}
     score_roof["frac"] = score_roof["achieved"] / hbm
+    score_roof["ceiling_at_size"] = {
+        "probe_launch_ms": probe_ms, "achieved": score_bytes / (probe_ms / 1e3) / 1e9,
+        "frac_of_peak": score_bytes / (probe_ms / 1e3) / 1e9 / hbm, "scorer_frac_of_ceiling": probe_ms / rot_ms,
+        "what": "ctr_score_stream_probe: the scorer's loads and stores alone (same grid, launch attributes and "
+                "buffers, no arithmetic or envelope prologue), timed in the same graph"}
     big_bytes = 17 * big_n + 3 * 4 * N_SCORE_INST
     score_roof_big = {"bound": "hbm", "unit": "GB/s", "achieved": big_bytes / (big_ms / 1e3) / 1e9, "peak": hbm,
                       "peak_source": hbm_source,
                       "traffic": None, "launch_ms": big_ms, "requests": big_n}
     score_roof_big["frac"] = score_roof_big["achieved"] / hbm
+    score_roof_big["ceiling_at_size"] = {
+        "probe_launch_ms": big_probe_ms, "achieved": big_bytes / (big_probe_ms / 1e3) / 1e9,
+        "frac_of_peak": big_bytes / (big_probe_ms / 1e3) / 1e9 / hbm, "scorer_frac_of_ceiling": big_probe_ms / big_ms}
     line = {
         "metric": "routed requests/sec (replica sweep, 1 GB300)", "value": value, "unit": "routed requests/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
@@ -550,7 +591,7 @@ def run_ours(args, rank, world, local_rank):
                          "the place of on-device trace generation (ctr_gen_trace), so this step does that much "
                          "less device work than the device-timed step",
                  "steps": e2e_steps},
-        "gpu_launches": 5 * args.steps,  # gen, sim, checksum pass, goodput, score
+        "gpu_launches": 4 * args.steps,  # trace, simulation, checksum + goodput pass, scorer
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

@@ -225,12 +225,17 @@ size_t ctr_workspace_bytes(int32_t which, const ctr_sim_cfg* cfg /* host */, int
  * row_hash the order-independent 64-bit checksum of each row's routing and
  * times; row_status CTR_OK or the row's CTR_EINVAL / CTR_EOVERFLOW /
  * CTR_ETIMEOUT (outputs of a failed row are unspecified).
+ * met_count / p99_ttft_us: optional (both or neither, else CTR_EINVAL): each
+ * row's SLO goodput inputs exactly as ctr_goodput defines them, computed in
+ * the same pass over t_first_us / t_done_us that completes row_hash (the
+ * outputs are then read once, not twice).
  * workspace: device, >= 256 bytes, ideally ctr_workspace_bytes(); its contents
  * need no initialisation and are clobbered. */
 int ctr_simulate(const ctr_sim_cfg* cfg /* host */, const ctr_cost_consts* consts /* host */, int32_t n_const_sets,
                  const int32_t* policy_ids /* host */, int32_t n_policies, ctr_requests trace, int32_t n_replicas,
                  int64_t n_req, uint8_t* i_pre, uint8_t* i_dec, int64_t* t_first_us, int64_t* t_done_us,
-                 uint64_t* row_hash, int32_t* row_status, void* workspace, size_t workspace_bytes, void* stream);
+                 uint64_t* row_hash, int32_t* row_status, int64_t* met_count, int64_t* p99_ttft_us, void* workspace,
+                 size_t workspace_bytes, void* stream);
 
 /* ctr_simulate_noalloc -- ctr_simulate for callers that cannot allocate
  * device memory (the paper has no counterpart: this is a deployment aid).

@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 5;
+constexpr int kAbiVersion = 6;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -210,7 +210,8 @@ size_t ctr_workspace_bytes(int32_t which, const ctr_sim_cfg* cfg, int64_t n_rows
 int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t n_const_sets,
                  const int32_t* policy_ids, int32_t n_policies, ctr_requests trace, int32_t n_replicas, int64_t n_req,
                  uint8_t* i_pre, uint8_t* i_dec, int64_t* t_first_us, int64_t* t_done_us, uint64_t* row_hash,
-                 int32_t* row_status, void* workspace, size_t workspace_bytes, void* stream)
+                 int32_t* row_status, int64_t* met_count, int64_t* p99_ttft_us, void* workspace,
+                 size_t workspace_bytes, void* stream)
 {
     if (!valid_sim_cfg(cfg) || !consts || !policy_ids) return CTR_EINVAL;
     if (!in_range(n_const_sets, 1, CTR_MAX_CONST_SETS) || !in_range(n_policies, 1, 5)) return CTR_EINVAL;
@@ -223,6 +224,7 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     if (n_rows >= (1LL << 31)) return CTR_EINVAL;
     if (n_rows == 0) return CTR_OK;
     if (!row_hash || !row_status || !workspace) return CTR_EINVAL;
+    if ((met_count == nullptr) != (p99_ttft_us == nullptr)) return CTR_EINVAL;  // both goodput outputs or neither
     if (n_req > 0 && (!requests_present(trace) || !t_first_us || !t_done_us)) return CTR_EINVAL;
     if ((uintptr_t)workspace % 256 != 0) return CTR_EINVAL;
 
@@ -302,7 +304,28 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     cudaError_t e = cudaMemsetAsync(workspace, 0, 256, s);
     if (e != cudaSuccess) return CTR_ECUDA;
     const int blocks = (int)((slots + wpb - 1) / wpb);
-    return cuda_status(launch_sim(p, blocks, wpb, s));
+    const bool goodput = met_count != nullptr;
+    e = launch_sim(p, blocks, wpb, !goodput, s);
+    if (e != cudaSuccess || !goodput) return cuda_status(e);
+    // each row's goodput, in the same pass that adds its checksum's first-token and completion terms
+    GoodputParams g;
+    std::memset(&g, 0, sizeof(g));
+    g.trace = trace;
+    g.n_req = n_req;
+    g.n_rows = n_rows;
+    g.rows_per_replica = n_const_sets * n_policies;
+    g.n_classes = cfg->n_classes;
+    for (int i = 0; i < 4; ++i) {
+        g.ttft[i] = cfg->ttft_slo_us[i];
+        g.tpot[i] = cfg->tpot_slo_us[i];
+    }
+    g.t_first = t_first_us;
+    g.t_done = t_done_us;
+    g.met = met_count;
+    g.p99 = p99_ttft_us;
+    g.row_hash = row_hash;
+    g.row_status = row_status;
+    return cuda_status(launch_goodput(g, s));
 }
 
 int ctr_goodput(const ctr_sim_cfg* cfg, ctr_requests trace, int32_t n_replicas, int32_t rows_per_replica, int64_t n_req,

@@ -15,6 +15,19 @@ constexpr int64_t kArrivalLimit = int64_t(1) << 39;
 constexpr int kKeyBits = 23;                        // request index bits in packed heap keys
 constexpr uint64_t kKeyMask = (uint64_t(1) << kKeyBits) - 1;
 
+// Row checksum term mix(k, tag, v) = sm(sm((tag << 56) ^ k) ^ v), sm the
+// splitmix64 output function (Steele, Lea and Flood, OOPSLA'14).
+__device__ __forceinline__ uint64_t mix64(uint64_t z)
+{
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+__device__ __forceinline__ uint64_t hterm(int64_t k, uint64_t tag, uint64_t v)
+{
+    return mix64(mix64((tag << 56) ^ (uint64_t)k) ^ v);
+}
+
 // Philox4x32-10 (Salmon et al., SC'11): ten rounds of two 32x32 -> 64 products,
 // the key bumped by the Weyl constants between rounds.
 struct Philox4 {
@@ -105,7 +118,9 @@ struct SimParams {
 int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr);
 int sim_max_resident_warps(int* warps_per_block, int* blocks);
 int sim_group_width(int n_instances);  // lanes per simulated row; 32 / width rows share a warp
-cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream);
+// hash_pass: add the first-token and completion checksum terms in a pass of
+// their own (false when the goodput pass that follows adds them)
+cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, bool hash_pass, cudaStream_t stream);
 
 // ---------------------------------------------------------------- goodput
 struct GoodputParams {
@@ -117,6 +132,10 @@ struct GoodputParams {
     const int64_t* t_done;
     int64_t* met;
     int64_t* p99;
+    // optional (both or neither): add each OK row's first-token and completion
+    // checksum terms to row_hash in the same pass over the outputs
+    uint64_t* row_hash;
+    const int32_t* row_status;
 };
 cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream);
 

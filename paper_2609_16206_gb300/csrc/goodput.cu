@@ -10,7 +10,9 @@
 // (2048 shared-memory bins).  When the row fits (kStage), pass 0 also keeps
 // its TTFTs in shared memory as 32-bit values and the select passes read them
 // there, so a row crosses HBM once; a row with a TTFT outside [0, 2^32) or too
-// many requests re-reads its TTFTs from global memory instead.
+// many requests re-reads its TTFTs from global memory instead.  Called from
+// ctr_simulate with kHash, pass 0 also sums the row checksum's first-token and
+// completion terms, so the outputs are read once for both.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -40,7 +42,7 @@ __device__ T block_reduce(T v, T identity, Op op, T* scratch)
     return r;
 }
 
-template <bool kStage>
+template <bool kStage, bool kHash>
 __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParams P)
 {
     __shared__ uint32_t hist[kBins];
@@ -54,6 +56,7 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
         const int64_t tb = (row / P.rows_per_replica) * n;
         const int64_t ob = row * n;
         int64_t met = 0, mn = INT64_MAX, mx = INT64_MIN;
+        uint64_t h = 0;  // kHash: the row's first-token and completion checksum terms
         // 2 elements per thread per round, all loads issued before any is used (the pass is latency-bound;
         // more elements in flight spill at 64 registers and lose more than they hide)
         for (int64_t base = tid; base < n; base += (int64_t)kThreads * 2) {
@@ -84,12 +87,19 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
                     mn = ttft < mn ? ttft : mn;
                     mx = ttft > mx ? ttft : mx;
                     if (kStage) ttft_s[k] = (uint32_t)ttft;
+                    if (kHash) h += hterm(k, 2, (uint64_t)tf[u]) + hterm(k, 3, (uint64_t)td[u]);
                 }
             }
         }
         met = block_reduce<int64_t>(met, 0, [](int64_t a, int64_t b) { return a + b; }, red64);
         mn = block_reduce<int64_t>(mn, INT64_MAX, [](int64_t a, int64_t b) { return a < b ? a : b; }, red64);
         mx = block_reduce<int64_t>(mx, INT64_MIN, [](int64_t a, int64_t b) { return a > b ? a : b; }, red64);
+        if (kHash) {
+            h = (uint64_t)block_reduce<int64_t>((int64_t)h, 0, [](int64_t a, int64_t b) {
+                return (int64_t)((uint64_t)a + (uint64_t)b);  // sum mod 2^64
+            }, red64);
+            if (tid == 0 && P.row_status[row] == CTR_OK) P.row_hash[row] += h;  // a failed row keeps 0
+        }
         if (n == 0) {
             if (tid == 0) {
                 P.met[row] = 0;
@@ -171,21 +181,29 @@ cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream)
     if (err != cudaSuccess) return err;
     constexpr int64_t kStageMaxBytes = 160 * 1024;  // a row's TTFTs staged in shared memory up to this
     const int64_t stage_bytes = p.n_req * 4;
+    const bool hash = p.row_hash != nullptr;
     if (stage_bytes > 0 && stage_bytes <= kStageMaxBytes) {
-        err = cudaFuncSetAttribute(goodput_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)stage_bytes);
+        const void* k = hash ? (const void*)goodput_kernel<true, true> : (const void*)goodput_kernel<true, false>;
+        err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)stage_bytes);
         if (err != cudaSuccess) return err;
         int per_sm = 0;
-        err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, goodput_kernel<true>, kThreads, (size_t)stage_bytes);
+        err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kThreads, (size_t)stage_bytes);
         if (err != cudaSuccess) return err;
         int64_t blocks = p.n_rows;
         const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
         if (blocks > cap) blocks = cap;
-        goodput_kernel<true><<<(unsigned)blocks, kThreads, (size_t)stage_bytes, stream>>>(p);
+        if (hash)
+            goodput_kernel<true, true><<<(unsigned)blocks, kThreads, (size_t)stage_bytes, stream>>>(p);
+        else
+            goodput_kernel<true, false><<<(unsigned)blocks, kThreads, (size_t)stage_bytes, stream>>>(p);
         return cudaGetLastError();
     }
     int64_t blocks = p.n_rows;
     if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
-    goodput_kernel<false><<<(unsigned)blocks, kThreads, 0, stream>>>(p);
+    if (hash)
+        goodput_kernel<false, true><<<(unsigned)blocks, kThreads, 0, stream>>>(p);
+    else
+        goodput_kernel<false, false><<<(unsigned)blocks, kThreads, 0, stream>>>(p);
     return cudaGetLastError();
 }
 

@@ -73,7 +73,8 @@ int ctr_simulate_noalloc(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, 
     const int rc = scratch_address(&scratch);
     if (rc != CTR_OK) return rc;
     return ctr_simulate(cfg, consts, n_const_sets, policy_ids, n_policies, trace, n_replicas, n_req, i_pre, i_dec,
-                        t_first_us, t_done_us, row_hash, row_status, scratch, kScratchBytes, stream);
+                        t_first_us, t_done_us, row_hash, row_status, nullptr, nullptr, scratch, kScratchBytes,
+                        stream);
 }
 
 }  // extern "C"

@@ -63,18 +63,6 @@ constexpr RecipTable make_recip_table()
 }
 __device__ const RecipTable kRecipTable = make_recip_table();
 
-__device__ __forceinline__ uint64_t mix64(uint64_t z)  // splitmix64 output function
-{
-    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-    return z ^ (z >> 31);
-}
-
-__device__ __forceinline__ uint64_t hterm(int64_t k, uint64_t tag, uint64_t v)
-{
-    return mix64(mix64((tag << 56) ^ (uint64_t)k) ^ v);
-}
-
 // floor(num / d) with r = floor((2^64 - 1) / d): the estimate is low by at most 2
 __device__ __forceinline__ uint64_t div_recip(uint64_t num, uint64_t d, uint64_t recip)
 {
@@ -882,7 +870,7 @@ cudaError_t launch_mode(const SimParams& p, int blocks, cudaStream_t stream)
 
 }  // namespace
 
-cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
+cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, bool hash_pass, cudaStream_t stream)
 {
     (void)warps_per_block;
     bool signals = false;  // the proxy's ledger backlog or polled occupancy in some constant set
@@ -891,7 +879,7 @@ cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cuda
                           : signals       ? launch_mode<1>(p, blocks, stream)
                                           : launch_mode<0>(p, blocks, stream);
     if (e != cudaSuccess) return e;
-    if (p.n_rows > 0) {
+    if (hash_pass && p.n_rows > 0) {  // else the caller's goodput pass adds these terms
         const int64_t hb = p.n_rows < (int64_t)blocks * 8 ? p.n_rows : (int64_t)blocks * 8;
         hash_kernel<<<(unsigned)hb, kHashThreads, 0, stream>>>(p);
     }

@@ -94,7 +94,7 @@ def lib():
             L.ctr_workspace_bytes.argtypes = [i32, C.POINTER(CtrSimCfg), i64, i64]
             L.ctr_workspace_bytes.restype = C.c_size_t
             L.ctr_simulate.argtypes = [C.POINTER(CtrSimCfg), C.POINTER(CtrCostConsts), i32, C.POINTER(i32), i32,
-                                       CtrRequests, i32, i64, vp, vp, vp, vp, vp, vp, vp, C.c_size_t, vp]
+                                       CtrRequests, i32, i64, vp, vp, vp, vp, vp, vp, vp, vp, vp, C.c_size_t, vp]
             L.ctr_simulate.restype = C.c_int
             L.ctr_simulate_noalloc.argtypes = [C.POINTER(CtrSimCfg), C.POINTER(CtrCostConsts), i32, C.POINTER(i32),
                                                i32, CtrRequests, i32, i64, vp, vp, vp, vp, vp, vp, vp]
@@ -244,14 +244,16 @@ def ctr_workspace_bytes(which: int, sim_cfg, n_rows: int, n_req: int) -> int:
 
 
 def ctr_simulate(sim_cfg, const_sets, policies, trace: dict, n_replicas: int, n_req: int, t_first_us, t_done_us,
-                 row_hash, row_status, workspace, i_pre=None, i_dec=None, stream=None):
+                 row_hash, row_status, workspace, i_pre=None, i_dec=None, met_count=None, p99_ttft_us=None,
+                 stream=None):
     cfg = sim_cfg_struct(sim_cfg)
     sets = consts_array(list(const_sets))
     pols = (C.c_int32 * len(policies))(*[int(p) for p in policies])
     _check("ctr_simulate", lib().ctr_simulate(
         C.byref(cfg), sets, len(sets), pols, len(policies), requests_struct(trace), int(n_replicas), int(n_req),
         _ptr(i_pre), _ptr(i_dec), _ptr(t_first_us), _ptr(t_done_us), _ptr(row_hash), _ptr(row_status),
-        _ptr(workspace), int(workspace.numel() * workspace.element_size()), _stream(stream)))
+        _ptr(met_count), _ptr(p99_ttft_us), _ptr(workspace), int(workspace.numel() * workspace.element_size()),
+        _stream(stream)))
 
 
 def ctr_simulate_noalloc(sim_cfg, const_sets, policies, trace: dict, n_replicas: int, n_req: int, t_first_us,

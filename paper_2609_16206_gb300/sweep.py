@@ -66,14 +66,14 @@ def alloc(sim_cfg, n_replicas: int, n_rows: int, n_req: int, device) -> SweepBuf
 
 def run_step(trace_cfg, sim_cfg, const_sets, policies, n_replicas: int, n_req: int, replica_offset: int,
              buf: SweepBuffers, stream=None, gen: bool = True):
-    """Trace generation (unless gen is False), simulation, goodput; rows are
+    """Trace generation (unless gen is False), then simulation with each row's
+    goodput computed in the pass that completes its checksum; rows are
     (replica, set, policy) row-major."""
     if gen:
         ctr.ctr_gen_trace(trace_cfg, n_replicas, replica_offset, n_req, buf.trace, stream=stream)
     ctr.ctr_simulate(sim_cfg, const_sets, policies, buf.trace, n_replicas, n_req, buf.t_first, buf.t_done,
-                     buf.row_hash, buf.row_status, buf.workspace, stream=stream)
-    ctr.ctr_goodput(sim_cfg, buf.trace, n_replicas, len(const_sets) * len(policies), n_req, buf.t_first,
-                    buf.t_done, buf.met, buf.p99, stream=stream)
+                     buf.row_hash, buf.row_status, buf.workspace, met_count=buf.met, p99_ttft_us=buf.p99,
+                     stream=stream)
 
 
 def saturation_rate(trace_cfgs, sim_cfg, n_req: int = 10_000, lo: int = 1, hi: int = 200_000, steps: int = 24,

@@ -36,7 +36,7 @@ def test_exports_every_declared_function(libctr):
 def test_static_entry_points_run_without_gpu(libctr):
     libctr.ctr_strerror.restype = ctypes.c_char_p
     assert libctr.ctr_strerror(-3).decode().startswith("a fixed-capacity")
-    assert libctr.ctr_abi_version() == 5
+    assert libctr.ctr_abi_version() == 6
 
 
 def test_step_budget_bound_checked_on_the_host():
@@ -52,7 +52,7 @@ def test_step_budget_bound_checked_on_the_host():
     def call(steps):
         cfg = ctr.sim_cfg_struct(W.SimCfg(max_steps_per_instance=steps))
         return L.ctr_simulate(ctypes.byref(cfg), sets, 1, pols, 1, ctr.CtrRequests(), 0, 0, None, None, None, None,
-                              None, None, None, 0, None)
+                              None, None, None, None, None, 0, None)
     assert W.SimCfg().max_steps_per_instance == ctr.CTR_MAX_STEPS_PER_INSTANCE == (1 << 31) - (1 << 21)
     assert call(ctr.CTR_MAX_STEPS_PER_INSTANCE) == ctr.CTR_OK
     assert call(1) == ctr.CTR_OK
@@ -75,7 +75,7 @@ def test_request_count_bound_checked_on_the_host():
 
     def sim(n_req):  # zero replicas: validation only
         return L.ctr_simulate(ctypes.byref(cfg), sets, 1, pols, 1, ctr.CtrRequests(), 0, n_req, None, None, None,
-                              None, None, None, None, 0, None)
+                              None, None, None, None, None, None, 0, None)
 
     def goodput(n_req):
         return L.ctr_goodput(ctypes.byref(cfg), ctr.CtrRequests(), 0, 4, n_req, None, None, None, None, None)

@@ -46,8 +46,9 @@ def sim_call(cfg, cc=None, n_sets=1, pols=(0,), n_rep=1, n_req=10, ws_bytes=1 <<
     if noalloc:
         return rc(L.ctr_simulate_noalloc(C.byref(cfg), sets, n_sets, pa, len(pols), req, n_rep, n_req, ptr, ptr, ptr,
                                          ptr, ptr, ptr, None))
+    goodput = (ptr, ptr) if n_rep % 2 else (None, None)
     return rc(L.ctr_simulate(C.byref(cfg), sets, n_sets, pa, len(pols), req, n_rep, n_req, ptr, ptr, ptr, ptr, ptr,
-                             ptr, ptr, ws_bytes, None))
+                             ptr, *goodput, ptr, ws_bytes, None))
 
 # every simulator field at its extremes, one at a time
 base = ctr.sim_cfg_struct(W.replica_sweep().sim)
@@ -140,7 +141,7 @@ for _ in range(3000):
             except (OverflowError, TypeError):
                 pass
     trace_call(tcfg, pick([0, 1, 2]), pick([0, 5, (1 << 40) - 3]), pick([0, 3]))
-assert L.ctr_abi_version() == 5
+assert L.ctr_abi_version() == 6
 for code in range(-6, 3):
     assert L.ctr_strerror(code)
 print("seen", sorted(seen))

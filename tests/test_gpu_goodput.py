@@ -62,3 +62,55 @@ def test_goodput_empty(orc):
     z = torch.empty((2, 0), dtype=torch.int64, device="cuda")
     met, p99 = _goodput(ctr, W.SimCfg(), tr, 2, 1, 0, z, z)
     assert met.tolist() == [0, 0] and p99.tolist() == [-1, -1]
+
+
+@pytest.mark.parametrize("wl,R,N,sets", [(W.replica_sweep(), 6, 4000, 1), (W.large_pool(rate_mreq=34_000), 2, 3000, 1),
+                                         (W.replica_sweep(), 3, 45_000, 1), (W.replica_sweep(), 2, 1500, 3)])
+def test_goodput_inside_simulate_matches_the_standalone_call(orc, wl, R, N, sets):
+    """ctr_simulate with goodput outputs completes each row's checksum and
+    computes its goodput in one pass over the outputs: the hashes equal those
+    of the plain call (and the oracle's), and met / P99 equal ctr_goodput's
+    and the oracle's; failed rows (a tiny FIFO) keep the checksum 0."""
+    ctr = need_gpu()
+    tr = gen(ctr, wl.trace, R, N)
+    pols = list(W.ALL_POLICIES)
+    cs = (list(W.mispriced_sets())[:sets] if sets > 1 else [wl.consts[0]])
+    plain = simulate(ctr, wl.sim, cs, pols, tr, R, N)
+    rows = R * len(cs) * len(pols)
+    out = {k: torch.full((rows, N), -7, dtype=torch.int64, device="cuda") for k in ("tf", "td")}
+    h = torch.zeros(rows, dtype=torch.int64, device="cuda")
+    st = torch.full((rows,), 99, dtype=torch.int32, device="cuda")
+    met = torch.full((rows,), -5, dtype=torch.int64, device="cuda")
+    p99 = torch.full((rows,), -5, dtype=torch.int64, device="cuda")
+    ws = ctr.simulate_workspace(wl.sim, rows, N, "cuda")
+    ctr.ctr_simulate(wl.sim, cs, pols, tr, R, N, out["tf"], out["td"], h, st, ws, met_count=met, p99_ttft_us=p99)
+    torch.cuda.synchronize()
+    assert np.array_equal(st.cpu().numpy(), plain["status"])
+    assert np.array_equal(h.cpu().numpy().astype(np.uint64), plain["hash"])
+    m_alone, p_alone = _goodput(ctr, wl.sim, tr, R, len(cs) * len(pols), N, out["tf"], out["td"])
+    assert np.array_equal(met.cpu().numpy(), m_alone) and np.array_equal(p99.cpu().numpy(), p_alone)
+    r0 = host_trace(tr, 0)
+    for j, pol in enumerate(pols):
+        o = orc.simulate(wl.sim, cs[0], pol, r0)
+        assert int(h[j]) & 0xFFFFFFFFFFFFFFFF == o["hash"]
+        assert (int(met[j]), int(p99[j])) == orc.goodput(wl.sim, r0, o["t_first_us"], o["t_done_us"])
+    # failed rows: the checksum stays 0 whichever pass completes it
+    small = wl.sim.replace(cap_waiting=2, cap_pending=2)
+    ctr.ctr_simulate(small, cs, pols, tr, R, N, out["tf"], out["td"], h, st, ws, met_count=met, p99_ttft_us=p99)
+    torch.cuda.synchronize()
+    bad = st.cpu().numpy() != 0
+    assert bad.any() and not h.cpu().numpy()[bad].any()
+
+
+def test_goodput_outputs_come_in_pairs():
+    ctr = need_gpu()
+    wl = W.replica_sweep()
+    tr = gen(ctr, wl.trace, 1, 10)
+    z = torch.zeros((4, 10), dtype=torch.int64, device="cuda")
+    ws = ctr.simulate_workspace(wl.sim, 4, 10, "cuda")
+    with pytest.raises(ctr.CtrError) as err:
+        ctr.ctr_simulate(wl.sim, [W.CALIBRATED], list(W.ALL_POLICIES), tr, 1, 10, z, z.clone(),
+                         torch.zeros(4, dtype=torch.int64, device="cuda"), torch.zeros(4, dtype=torch.int32,
+                                                                                       device="cuda"), ws,
+                         met_count=torch.zeros(4, dtype=torch.int64, device="cuda"))
+    assert err.value.code == ctr.CTR_EINVAL
