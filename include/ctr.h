@@ -187,7 +187,8 @@ int ctr_gen_trace(const ctr_trace_cfg* cfg /* host */, int32_t n_replicas, int64
  * its fp32 cost; a slo_class >= 4 gives -1 and NaN.  Inputs must be finite and
  * non-negative.  n_req >= 0, 1 <= n_inst <= CTR_SCORE_MAX_INST.  status is an
  * optional device int32 (NULL ok) set to CTR_ETIMEOUT if the shared-memory
- * staging wait of a block ran past its bound (never expected).
+ * staging wait of a block ran past its bound (never expected); that block then
+ * scores nothing, so out_argmin and out_cost are unspecified for the call.
  * The kernel is launched as a programmatic dependent launch: it reads nothing
  * before the preceding work in the stream has completed, and it lets a
  * following kernel launched the same way be scheduled while it drains (such a

@@ -314,24 +314,26 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
 
     if (bulk) {
         __syncthreads();  // the barrier is initialised before any thread polls it
-        uint32_t done = 0;
-        for (unsigned it = 0; it < kWaitLimit && !done; ++it) {
-            asm volatile(
-                "{\n\t.reg .pred p;\n\t"
-                "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n\t"
-                "selp.u32 %0, 1, 0, p;\n\t}"
-                : "=r"(done)
-                : "r"(bar)
-                : "memory");
-        }
-        if (__syncthreads_or(!done)) {  // block-uniform decision
-            // never expected: report it and read the state with plain loads instead
-            if (tid == 0 && P.status) atomicExch(P.status, CTR_ETIMEOUT);
-            for (int d = tid; d < n_inst; d += kThreads) {
-                sm.q[d] = P.Q[d];
-                sm.a[d] = P.A[d];
-                sm.kap[d] = P.kap[d];
+        auto staged = [&]() {  // bounded polling of the staging barrier
+            uint32_t done = 0;
+            for (unsigned it = 0; it < kWaitLimit && !done; ++it) {
+                asm volatile(
+                    "{\n\t.reg .pred p;\n\t"
+                    "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n\t"
+                    "selp.u32 %0, 1, 0, p;\n\t}"
+                    : "=r"(done)
+                    : "r"(bar)
+                    : "memory");
             }
+            return done != 0;
+        };
+        if (__syncthreads_or(!staged())) {  // block-uniform decision
+            // never expected: report it, give the copies in flight a second bounded wait
+            // (the block must not leave with them still writing its shared memory),
+            // and score nothing: the call's outputs are unspecified
+            if (tid == 0 && P.status) atomicExch(P.status, CTR_ETIMEOUT);
+            (void)__syncthreads_or(!staged());
+            return;
         }
     } else {
         for (int d = tid; d < n_inst; d += kThreads) {

@@ -169,8 +169,12 @@ __device__ __forceinline__ int warp_argmin(uint64_t v)
     return __ffs(ball) - 1;
 }
 
+// A decode lane's state.  `sum` is the one in-flight sum the row's policy
+// reads: the true remaining output tokens R for the learned router on the true
+// backlog, the predicted lengths o_hat for the length heuristic and the proxy's
+// ledger (sum_is_o_hat), nothing for the others.
 struct Decode {
-    int64_t step_end, R, ohat;
+    int64_t step_end, sum;
     int32_t step_idx;        // steps ended; the step budget keeps it and every completion step below 2^31
     int32_t kv_res, kv_rsv;  // resident <= reserved <= C < 2^31 tokens
     uint64_t pend_top, act_top;
@@ -203,7 +207,7 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
 template <bool kSnap>
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
                                               uint32_t* wait, int64_t tb, int64_t ob, int64_t& tsnap, int64_t& kv_snap,
-                                              bool track_ohat)
+                                              bool sum_is_o_hat)
 {
     for (;;) {
         // Plain step ends first: the step ends by T, no request finishes with
@@ -253,7 +257,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             const int64_t mn = (int64_t)m * n;
             s.step_idx += m;
             s.kv_res += (int32_t)mn;  // stays within the reservation
-            s.R -= mn;
+            if (!sum_is_o_hat) s.sum -= mn;  // R: every active request is one token closer
             if (s.step_idx >= (int32_t)P.max_steps) return CTR_ETIMEOUT;
             s.step_end += (int64_t)m * S;
             if (s.step_end >= kTimeLimit) return CTR_EOVERFLOW;
@@ -272,7 +276,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
         if (s.stepping) {  // (1) the running step ends: one token for every active request
             s.step_idx += 1;
             s.kv_res += s.n_act;
-            s.R -= s.n_act;
+            if (!sum_is_o_hat) s.sum -= s.n_act;
             s.stepping = false;
             while (s.n_act > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
                 const int64_t k = (int64_t)(s.act_top & kKeyMask);
@@ -282,7 +286,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 s.q -= 1;
                 s.kv_res -= (int32_t)(pk + ok);
                 s.kv_rsv -= (int32_t)(pk + ok);
-                if (track_ohat) s.ohat -= __ldg(&P.trace.pred_out[tb + k]);
+                if (sum_is_o_hat) s.sum -= __ldg(&P.trace.pred_out[tb + k]);
                 P.t_done[ob + k] = tev;
             }
         }
@@ -421,8 +425,10 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         const int set = has_row ? (int)((row / P.n_pols) % P.n_sets) : 0;
         const int pol = has_row ? P.pols[row % P.n_pols] : CTR_POLICY_ROUND_ROBIN;
         const ConstsDev& cc = P.sets[set];
-        // the in-flight sum of predicted lengths is read only by the length heuristic and the proxy's ledger
-        const bool track_ohat = kSig || pol == CTR_POLICY_LENGTH_HEURISTIC;
+        // the in-flight sum the row's decode pricing reads: predicted lengths for the length
+        // heuristic and the proxy's ledger, else true remaining tokens (unread by JSQ / RR)
+        const bool learned_row = pol == CTR_POLICY_LEARNED || pol == CTR_POLICY_LEARNED_P2;
+        const bool sum_is_o_hat = pol == CTR_POLICY_LENGTH_HEURISTIC || (kSig && learned_row && cc.proxy);
         const int64_t tb = rep * n;
         const int64_t ob = row * n;
 
@@ -437,15 +443,15 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         bool live = has_row && valid;
 
         Decode s;
-        s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.R = 0; s.ohat = 0;
+        s.step_end = 0; s.step_idx = 0; s.kv_res = 0; s.kv_rsv = 0; s.sum = 0;
         s.pend_top = kEmpty; s.act_top = kEmpty;
         s.n_act = 0; s.q = 0; s.pend_n = 0; s.w_head = 0; s.w_n = 0;
         s.stepping = false;
         // A lane simulates a prefill or a decode instance, never both, so a prefill
         // lane keeps its state in decode fields it does not use (fewer live registers).
         int64_t& busy = s.step_end;    // end of the last prefill (of the running batch, when batched)
-        int64_t& ring_front = s.ohat;  // the ring's front entry (end << 21 | p), read while ring_n > 0
-        int64_t& ring_sum_p = s.R;     // prompt tokens of the prefills in the ring
+        uint64_t& ring_front = s.act_top;  // the ring's front entry (end << 21 | p), read while ring_n > 0
+        int64_t& ring_sum_p = s.sum;       // prompt tokens of the prefills in the ring
         int32_t& ring_head = s.w_head;
         int32_t& ring_n = s.w_n;
         int64_t kv_seen = 0, last_poll = -1;     // decode lanes: occupancy at the last poll instant
@@ -556,14 +562,14 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 last_poll = tp;
                             }
                         }
-                        if (err == CTR_OK) err = decode_advance<kSig>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen, track_ohat);
+                        if (err == CTR_OK) err = decode_advance<kSig>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen, sum_is_o_hat);
                     } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
-                        while (ring_n > 0 && ring_front <= thr) {
+                        while (ring_n > 0 && ring_front <= (uint64_t)thr) {
                             if constexpr (kSig) ring_sum_p -= ring_front & kRingPMask;
                             ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
                             ring_n -= 1;
-                            ring_front = ring_n > 0 ? ring[ring_head] : kNever;
+                            ring_front = ring_n > 0 ? (uint64_t)ring[ring_head] : (uint64_t)kNever;
                         }
                         if (ring_n == 0) ring_head = 0;
                     }
@@ -606,8 +612,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         if (learned) {
                             const int64_t na = s.n_act;
                             const int64_t step = P.dec_base + (int64_t)(int32_t)P.dec_seq * s.n_act + kv_term(s.kv_res, P);
-                            const uint64_t hi = __umul64hi((uint64_t)s.R, (uint64_t)step);
-                            const uint64_t lo = (uint64_t)s.R * (uint64_t)step;
+                            const uint64_t hi = __umul64hi((uint64_t)s.sum, (uint64_t)step);
+                            const uint64_t lo = (uint64_t)s.sum * (uint64_t)step;
                             int64_t b;
                             if (hi != 0 || lo >= (1ull << 62)) {
                                 b = kBacklogClamp;
@@ -618,7 +624,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
                             if (kSig && cc.proxy) {  // the ledger: tau_dec o_hat per request routed here and not done
-                                b = (cc.ablate & CTR_ABLATE_PREDICTED_LENGTH) ? 0 : cc.tau_dec * s.ohat;
+                                b = (cc.ablate & CTR_ABLATE_PREDICTED_LENGTH) ? 0 : cc.tau_dec * s.sum;
                                 if (b > kBacklogClamp) b = kBacklogClamp;
                             }
                             const int64_t kv = kSig && cc.poll_us > 0 ? kv_seen : s.kv_res;
@@ -631,7 +637,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                             const int64_t load = cc.w_b * b + cc.w_s * priced;
                             cost = (uint64_t)(load * sig + cc.w_q * (int64_t)s.q * 65536);
                         } else if (pol == CTR_POLICY_LENGTH_HEURISTIC && ohk >= P.heur_thresh) {
-                            cost = (uint64_t)s.ohat;
+                            cost = (uint64_t)s.sum;
                         } else {
                             cost = (uint64_t)s.q;
                         }
@@ -707,7 +713,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         if (pos >= P.cap_ring) pos -= P.cap_ring;
                         const int64_t e = (end << kRingPBits) | pk;
                         ring[pos] = e;
-                        if (ring_n == 0) ring_front = e;
+                        if (ring_n == 0) ring_front = (uint64_t)e;
                         ring_n += 1;
                         if constexpr (kSig) ring_sum_p += pk;
                     }
@@ -723,8 +729,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     } else {
                         if (ready >= 0) heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
                         s.q += 1;
-                        s.R += ok;
-                        if (track_ohat) s.ohat += ohk;
+                        s.sum += sum_is_o_hat ? ohk : ok;
                     }
                 }
                 if (gl == j) my_route = ((uint32_t)ip << 8) | (uint32_t)id;
@@ -747,7 +752,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         }
         if (live && is_dec) {
             int64_t no_snap = -1;
-            err = decode_advance<false>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, track_ohat);
+            err = decode_advance<false>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, sum_is_o_hat);
         }
 
 #pragma unroll
