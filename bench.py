@@ -604,17 +604,17 @@ def run_ours(args, rank, world, local_rank):
 # per routed request, keyed by a hash of the simulator's code: a stale entry
 # (the kernel changed since the counters were taken) reports null.
 SIM_SLICE_COUNTERS: dict = {
-    "5e60eff741639c91": {"warp_inst_per_routed": 34340675617 / 81_920_000,
-                         "thread_inst_per_warp_inst": 285008436021 / 34340675617,
-                         "dram_bytes_per_routed": (2.39e9 + 1.57e9) / 81_920_000,
+    "8d95302a87f8aff8": {"warp_inst_per_routed": 34196262584 / 81_920_000,
+                         "thread_inst_per_warp_inst": 281902365249 / 34196262584,
+                         "dram_bytes_per_routed": (2382569216 + 1571453440) / 81_920_000,
                          "slice": "ncu on one launch of 1,024 replicas x 20,000 requests x 4 policies "
-                                  "(81.92 M routed requests): 3.434e10 warp-instructions, 2.850e11 thread-"
-                                  "instructions, 2.39 GB DRAM read + 1.57 GB written"},
+                                  "(81.92 M routed requests): 3.420e10 warp-instructions, 2.819e11 thread-"
+                                  "instructions, 2.383 GB DRAM read + 1.571 GB written"},
 }
 
 # DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.
 SCORE_DRAM_PER_LAUNCH: dict = {
-    "7b76efe5e7e4728b": {"read": 9.49e6, "write": 0.0},
+    "55623de89a963cd4": {"read": 9480704.0, "write": 0.0},
 }
 
 
