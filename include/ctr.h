@@ -38,6 +38,7 @@ extern "C" {
 #define CTR_MAX_STEPS_PER_INSTANCE ((1LL << 31) - (1LL << 21)) /* bound on the decode-step budget */
 #define CTR_SCORE_N_CONST 13      /* length of the standalone scorer's constant vector */
 #define CTR_SCORE_MAX_INST 256    /* instances per standalone scoring call */
+#define CTR_SCORE_MAX_REQ (1LL << 40) /* requests per standalone scoring call */
 
 enum ctr_policy {
     CTR_POLICY_LEARNED = 0,          /* marginal-cost argmin, sec. III-A / Algorithm 1 */
@@ -185,7 +186,7 @@ int ctr_gen_trace(const ctr_trace_cfg* cfg /* host */, int32_t n_replicas, int64
  *   [w_b, w_s, w_q, rho, tau_pre0, tau_pre, tau_dec, tau_act, 1/C, sigma_0..sigma_3].
  * Per request r: out_argmin[r] = argmin_d (ties -> lowest d) and out_cost[r]
  * its fp32 cost; a slo_class >= 4 gives -1 and NaN.  Inputs must be finite and
- * non-negative.  n_req >= 0, 1 <= n_inst <= CTR_SCORE_MAX_INST.  status is an
+ * non-negative.  0 <= n_req <= CTR_SCORE_MAX_REQ, 1 <= n_inst <= CTR_SCORE_MAX_INST.  status is an
  * optional device int32 (NULL ok) set to CTR_ETIMEOUT if the shared-memory
  * staging wait of a block ran past its bound (never expected); that block then
  * scores nothing, so out_argmin and out_cost are unspecified for the call.
@@ -204,7 +205,7 @@ int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_
  * arithmetic, on the same grid with the same loads and stores, writing
  * out_argmin[r] = slo_class[r] and out_cost[r] = prompt_len[r] + pred_out[r].
  * Timed beside the scorer it gives the HBM throughput a kernel of this shape
- * reaches at that size.  n_req a multiple of 4; float arrays 16-byte aligned,
+ * reaches at that size.  n_req a multiple of 4, at most CTR_SCORE_MAX_REQ; float arrays 16-byte aligned,
  * slo_class 4-byte aligned (CTR_EINVAL otherwise). */
 int ctr_score_stream_probe(const float* prompt_len, const float* pred_out, const uint8_t* slo_class, int64_t n_req,
                            int32_t* out_argmin, float* out_cost, void* stream);

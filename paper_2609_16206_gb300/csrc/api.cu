@@ -148,7 +148,8 @@ int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_
                     const float* q_tokens, const float* n_active, const float* kv_occ, int32_t n_inst,
                     const float* consts, int32_t* out_argmin, float* out_cost, int32_t* status, void* stream)
 {
-    if (n_req < 0 || n_inst < 1 || n_inst > CTR_SCORE_MAX_INST || !consts) return CTR_EINVAL;
+    if (n_req < 0 || n_req > CTR_SCORE_MAX_REQ || n_inst < 1 || n_inst > CTR_SCORE_MAX_INST || !consts)
+        return CTR_EINVAL;
     if (!q_tokens || !n_active || !kv_occ) return CTR_EINVAL;
     if (n_req > 0 && (!prompt_len || !pred_out || !slo_class || !out_argmin || !out_cost)) return CTR_EINVAL;
     ScoreParams p;
@@ -174,7 +175,7 @@ int ctr_score_batch(const float* prompt_len, const float* pred_out, const uint8_
 int ctr_score_stream_probe(const float* prompt_len, const float* pred_out, const uint8_t* slo_class, int64_t n_req,
                            int32_t* out_argmin, float* out_cost, void* stream)
 {
-    if (n_req < 0 || n_req % 4 != 0) return CTR_EINVAL;
+    if (n_req < 0 || n_req > CTR_SCORE_MAX_REQ || n_req % 4 != 0) return CTR_EINVAL;
     if (n_req > 0 && (!prompt_len || !pred_out || !slo_class || !out_argmin || !out_cost)) return CTR_EINVAL;
     if ((((uintptr_t)prompt_len | (uintptr_t)pred_out | (uintptr_t)out_argmin | (uintptr_t)out_cost) % 16u) != 0 ||
         (uintptr_t)slo_class % 4u != 0)

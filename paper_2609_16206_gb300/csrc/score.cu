@@ -13,10 +13,12 @@
 // class walks the envelope from o_hat = 0 by gift wrapping (one warp argmin
 // per segment); wider pools use every thread (a Pareto test, the o_hat
 // interval on which each surviving line wins, and its rank).  Each segment
-// keeps its instance's cost terms in one 16-byte entry.  Requests stream with
-// 128-bit loads, software-pipelined two vectors ahead: the count of
-// breakpoints at or below o_hat (a binary search past 8 segments) gives the
-// argmin, whose fp32 cost is then evaluated from the full formula.  The work
+// keeps its instance's cost terms, sigma_s folded in, in one 16-byte entry.
+// Requests stream with 128-bit loads, software-pipelined two vectors ahead,
+// each block over an equal contiguous range: the count of breakpoints at or
+// below o_hat (4 or 7 compares, chosen per block from its longest envelope; a
+// binary search past 8 segments) gives the argmin, whose fp32 cost is then
+// evaluated from the full formula.  The work
 // per request is O(log envelope size) instead of O(instances), which keeps the
 // kernel on the HBM roofline.  One block per SM, so the envelope is built 152
 // times, not once per request tile.
@@ -41,7 +43,7 @@ struct __align__(16) Smem {
     int valid_tmp[4][kMaxInst];
     int pareto[4][kMaxInst];
     float seg_lo[4][kMaxInst];
-    float4 seg_e[4][kMaxInst];  // per segment: kappa, BK, WQA of its instance, and the index (as bits)
+    float4 seg_e[4][kMaxInst];  // per segment: sigma w_s kappa, sigma w_s, sigma BK + WQA, index (as bits)
     float4 brk[4][2];  // breakpoints 1..7 of each class (seg_lo[s][1..7]), +inf past the last
     int nseg[4];
     unsigned long long bar;
@@ -91,24 +93,26 @@ __device__ __forceinline__ ReqTerms req_terms(const ScoreParams& P, float p, flo
     return ReqTerms{g, toh * P.c[3]};
 }
 
-// the full cost at the segment's instance e = (kappa_d, BK_d, WQA_d, d)
-__device__ __forceinline__ float cost_at(const ScoreParams& P, ReqTerms r, int s, float4 e)
-{
-    const float own = fmaf(r.h, e.x, r.g);
-    return fmaf(P.c[9 + s], fmaf(P.c[1], own, e.y), e.z);
-}
+// The full cost at the segment's instance, e = (sigma_s w_s kappa_d, sigma_s w_s,
+// sigma_s BK_d + WQA_d, d): sigma_s w_s kappa_d H + sigma_s w_s G + sigma_s BK_d + WQA_d,
+// every term non-negative, each path at most 7 roundings of 2^-24.
+__device__ __forceinline__ float cost_at(ReqTerms r, float4 e) { return fmaf(e.x, r.h, fmaf(e.y, r.g, e.z)); }
 
-// the segment entry of instance d
-__device__ __forceinline__ float4 seg_entry(const Smem& sm, const ScoreParams& P, int d)
+// the segment entry of instance d in class s
+__device__ __forceinline__ float4 seg_entry(const Smem& sm, const ScoreParams& P, int s, int d)
 {
     const float A = sm.a[d];
-    return make_float4(sm.kap[d], P.c[0] * fmaf(P.c[5], sm.q[d], P.c[7] * A), P.c[2] * A, __int_as_float(d));
+    const float sig = P.c[9 + s];
+    const float sws = sig * P.c[1];
+    const float bk = P.c[0] * fmaf(P.c[5], sm.q[d], P.c[7] * A);
+    return make_float4(sws * sm.kap[d], sws, fmaf(sig, bk, P.c[2] * A), __int_as_float(d));
 }
 
-// wide: some class has more than 8 segments (block-uniform), so the segment is
-// found by binary search instead of the branch-free count over 8 breakpoints
+// kB = 4 or 8: every class has at most kB + 1 segments (block-uniform), and the
+// segment is the count of its padded breakpoints <= o_hat; kB = 0: binary search
+template <int kB>
 __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, float p, float oh, uint32_t s,
-                                          bool wide, int& arg, float& cost)
+                                          int& arg, float& cost)
 {
     if (s >= 4) {
         arg = -1;
@@ -116,10 +120,13 @@ __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, 
         return;
     }
     int seg;
-    if (!wide) {  // segments start at 0 and at the sorted breakpoints: count those <= o_hat
-        const float4 b0 = sm.brk[s][0], b1 = sm.brk[s][1];
-        seg = (int)(b0.x <= oh) + (int)(b0.y <= oh) + (int)(b0.z <= oh) + (int)(b0.w <= oh) + (int)(b1.x <= oh) +
-              (int)(b1.y <= oh) + (int)(b1.z <= oh);
+    if (kB > 0) {  // segments start at 0 and at the sorted breakpoints: count those <= o_hat
+        const float4 b0 = sm.brk[s][0];
+        seg = (int)(b0.x <= oh) + (int)(b0.y <= oh) + (int)(b0.z <= oh) + (int)(b0.w <= oh);
+        if (kB > 4) {
+            const float4 b1 = sm.brk[s][1];
+            seg += (int)(b1.x <= oh) + (int)(b1.y <= oh) + (int)(b1.z <= oh);
+        }
     } else {
         int lo = 0, span = sm.nseg[s];
         while (span > 1) {  // last segment whose left end is <= o_hat
@@ -131,7 +138,7 @@ __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, 
     }
     const float4 e = sm.seg_e[s][seg];
     arg = __float_as_int(e.w);
-    cost = cost_at(P, req_terms(P, p, oh), (int)s, e);
+    cost = cost_at(req_terms(P, p, oh), e);
 }
 
 // (intercept, slope, index) lexicographic order of envelope lines
@@ -240,17 +247,92 @@ __device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst,
     }
     if (lane < nseg) {
         sm.seg_lo[s][lane] = lo0;
-        sm.seg_e[s][lane] = seg_entry(sm, P, id0);
+        sm.seg_e[s][lane] = seg_entry(sm, P, s, id0);
     }
     if (lane + 32 < nseg) {
         sm.seg_lo[s][lane + 32] = lo1;
-        sm.seg_e[s][lane + 32] = seg_entry(sm, P, id1);
+        sm.seg_e[s][lane + 32] = seg_entry(sm, P, s, id1);
     }
     if (lane >= 1 && lane <= 8) {  // padded breakpoints for the branch-free segment count
         float* b = reinterpret_cast<float*>(&sm.brk[s][0]);
         b[lane - 1] = lane < nseg ? lo0 : inf;
     }
     if (lane == 0) sm.nseg[s] = nseg;
+}
+
+// A thread's request vectors (4 requests each): block b owns the contiguous
+// range [n_vec * b / blocks, n_vec * (b + 1) / blocks), so every block streams
+// the same number of vectors within one, and its threads take every
+// kThreads-th vector from the block's start; the current vector and the next
+// are loaded ahead of their use.
+struct ReqPipe {
+    int64_t v, end;
+    bool has, hn;
+    float4 pv, ov, pn, on;
+    uint32_t cv, cn;
+};
+
+__device__ __forceinline__ void pipe_start(ReqPipe& q, const ScoreParams& P, int64_t n_vec, int tid)
+{
+    const float4* p4 = reinterpret_cast<const float4*>(P.p);
+    const float4* o4 = reinterpret_cast<const float4*>(P.oh);
+    const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
+    q.v = n_vec * blockIdx.x / gridDim.x + tid;
+    q.end = n_vec * (blockIdx.x + 1) / gridDim.x;
+    q.pv = q.ov = q.pn = q.on = make_float4(0.f, 0.f, 0.f, 0.f);
+    q.cv = q.cn = 0;
+    q.has = q.v < q.end;
+    if (q.has) {
+        q.pv = ld_stream(p4 + q.v);
+        q.ov = ld_stream(o4 + q.v);
+        q.cv = ld_stream_u32(c4 + q.v);
+    }
+    q.hn = q.v + kThreads < q.end;
+    if (q.hn) {
+        q.pn = ld_stream(p4 + q.v + kThreads);
+        q.on = ld_stream(o4 + q.v + kThreads);
+        q.cn = ld_stream_u32(c4 + q.v + kThreads);
+    }
+}
+
+// score the thread's vectors, two ahead: vector v is priced while v + kThreads
+// and v + 2 kThreads load
+template <int kB>
+__device__ __forceinline__ void pipe_score(ReqPipe& q, const Smem& sm, const ScoreParams& P)
+{
+    const float4* p4 = reinterpret_cast<const float4*>(P.p);
+    const float4* o4 = reinterpret_cast<const float4*>(P.oh);
+    const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
+    int4* a4 = reinterpret_cast<int4*>(P.argmin);
+    float4* f4 = reinterpret_cast<float4*>(P.cost);
+    while (q.has) {
+        const int64_t vf = q.v + 2 * kThreads;
+        const bool hf = vf < q.end;
+        float4 pf = make_float4(0.f, 0.f, 0.f, 0.f), of = pf;
+        uint32_t cf = 0;
+        if (hf) {
+            pf = ld_stream(p4 + vf);
+            of = ld_stream(o4 + vf);
+            cf = ld_stream_u32(c4 + vf);
+        }
+        int4 ai;
+        float4 fc;
+        score_one<kB>(sm, P, q.pv.x, q.ov.x, q.cv & 0xFFu, ai.x, fc.x);
+        score_one<kB>(sm, P, q.pv.y, q.ov.y, (q.cv >> 8) & 0xFFu, ai.y, fc.y);
+        score_one<kB>(sm, P, q.pv.z, q.ov.z, (q.cv >> 16) & 0xFFu, ai.z, fc.z);
+        score_one<kB>(sm, P, q.pv.w, q.ov.w, q.cv >> 24, ai.w, fc.w);
+        __stcs(a4 + q.v, ai);
+        __stcs(f4 + q.v, fc);
+        q.v += kThreads;
+        q.has = q.hn;
+        q.pv = q.pn;
+        q.ov = q.on;
+        q.cv = q.cn;
+        q.hn = hf;
+        q.pn = pf;
+        q.on = of;
+        q.cn = cf;
+    }
 }
 
 template <bool kVec>
@@ -292,25 +374,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
 
     // the first two request vectors of this thread, in flight while the block builds its envelopes
     const int64_t nv = kVec ? (P.n >> 2) : 0;
-    const int64_t stride = (int64_t)gridDim.x * kThreads;
-    int64_t v = (int64_t)blockIdx.x * kThreads + tid;
-    bool has = kVec && v < nv;
-    const float4* p4 = reinterpret_cast<const float4*>(P.p);
-    const float4* o4 = reinterpret_cast<const float4*>(P.oh);
-    const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
-    float4 pv = make_float4(0.f, 0.f, 0.f, 0.f), ov = pv, pn = pv, on = pv;
-    uint32_t cv = 0, cn = 0;
-    if (has) {
-        pv = ld_stream(p4 + v);
-        ov = ld_stream(o4 + v);
-        cv = ld_stream_u32(c4 + v);
-    }
-    bool hn = kVec && v + stride < nv;
-    if (hn) {
-        pn = ld_stream(p4 + v + stride);
-        on = ld_stream(o4 + v + stride);
-        cn = ld_stream_u32(c4 + v + stride);
-    }
+    ReqPipe q;
+    pipe_start(q, P, nv, tid);
 
     if (bulk) {
         __syncthreads();  // the barrier is initialised before any thread polls it
@@ -418,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         for (int off = 1; off < tpp; off <<= 1) rank += __shfl_xor_sync(0xffffffffu, rank, off, tpp);
         if (valid && part == 0) {
             sm.seg_lo[es][rank] = lo;
-            sm.seg_e[es][rank] = seg_entry(sm, P, ed);
+            sm.seg_e[es][rank] = seg_entry(sm, P, es, ed);
             atomicAdd(&sm.nseg[es], 1);
         }
         __syncthreads();
@@ -434,7 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
                 }
             }
             sm.seg_lo[tid][0] = 0.0f;
-            sm.seg_e[tid][0] = seg_entry(sm, P, best);
+            sm.seg_e[tid][0] = seg_entry(sm, P, tid, best);
             sm.nseg[tid] = 1;
         }
         __syncthreads();
@@ -447,44 +512,22 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         __syncthreads();
     }
 
-    // ---- stream the requests (the first vector was loaded before the prologue)
-    const bool wide = sm.nseg[0] > 8 || sm.nseg[1] > 8 || sm.nseg[2] > 8 || sm.nseg[3] > 8;
+    // ---- stream the requests (the first vectors were loaded before the prologue); the
+    // segment search is chosen once per block from the longest envelope
+    int maxseg = sm.nseg[0];
+    for (int c = 1; c < 4; ++c) maxseg = sm.nseg[c] > maxseg ? sm.nseg[c] : maxseg;
     if (kVec) {
-        int4* a4 = reinterpret_cast<int4*>(P.argmin);
-        float4* f4 = reinterpret_cast<float4*>(P.cost);
-        while (has) {  // two vectors ahead: v is computed while v + stride and v + 2 stride load
-            const int64_t vf = v + 2 * stride;
-            const bool hf = vf < nv;
-            float4 pf = make_float4(0.f, 0.f, 0.f, 0.f), of = pf;
-            uint32_t cf = 0;
-            if (hf) {
-                pf = ld_stream(p4 + vf);
-                of = ld_stream(o4 + vf);
-                cf = ld_stream_u32(c4 + vf);
-            }
-            int4 ai;
-            float4 fc;
-            score_one(sm, P, pv.x, ov.x, cv & 0xFFu, wide, ai.x, fc.x);
-            score_one(sm, P, pv.y, ov.y, (cv >> 8) & 0xFFu, wide, ai.y, fc.y);
-            score_one(sm, P, pv.z, ov.z, (cv >> 16) & 0xFFu, wide, ai.z, fc.z);
-            score_one(sm, P, pv.w, ov.w, cv >> 24, wide, ai.w, fc.w);
-            __stcs(a4 + v, ai);
-            __stcs(f4 + v, fc);
-            v += stride;
-            has = hn;
-            pv = pn;
-            ov = on;
-            cv = cn;
-            hn = hf;
-            pn = pf;
-            on = of;
-            cn = cf;
-        }
+        if (maxseg <= 5)
+            pipe_score<4>(q, sm, P);
+        else if (maxseg <= 8)
+            pipe_score<8>(q, sm, P);
+        else
+            pipe_score<0>(q, sm, P);
         if (blockIdx.x == 0 && tid < (int)(P.n & 3)) {
             const int64_t i = (nv << 2) + tid;
             int ai;
             float fc;
-            score_one(sm, P, P.p[i], P.oh[i], P.cls[i], wide, ai, fc);
+            score_one<0>(sm, P, P.p[i], P.oh[i], P.cls[i], ai, fc);
             P.argmin[i] = ai;
             P.cost[i] = fc;
         }
@@ -492,7 +535,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         for (int64_t i = (int64_t)blockIdx.x * kThreads + tid; i < P.n; i += (int64_t)gridDim.x * kThreads) {
             int ai;
             float fc;
-            score_one(sm, P, P.p[i], P.oh[i], P.cls[i], wide, ai, fc);
+            score_one<0>(sm, P, P.p[i], P.oh[i], P.cls[i], ai, fc);
             P.argmin[i] = ai;
             P.cost[i] = fc;
         }
@@ -502,7 +545,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
 // The scorer's memory traffic without its arithmetic or prologue: the same
 // grid, launch attributes, 128-bit streaming loads two vectors ahead and
 // streaming stores, writing class and p + o_hat.  It measures the HBM ceiling
-// the scorer can reach at a given size.
+// the scorer can reach at a given size.  It takes the vectors in grid-stride
+// order, which streams faster on its own than the scorer's contiguous block
+// ranges, so the ceiling it gives is the stricter of the two.
 __global__ void __launch_bounds__(kThreads, 1) stream_probe_kernel(const ScoreParams P)
 {
     asm volatile("griddepcontrol.wait;" ::: "memory");

@@ -24,6 +24,7 @@ CTR_MAX_REQUESTS = 1 << 23
 CTR_MAX_STEPS_PER_INSTANCE = (1 << 31) - (1 << 21)
 CTR_SCORE_N_CONST = 13
 CTR_SCORE_MAX_INST = 256
+CTR_SCORE_MAX_REQ = 1 << 40
 CTR_WS_SIMULATE = 0
 
 REQUEST_FIELDS = (("arrival_us", torch.int64), ("prompt_len", torch.int32), ("true_out", torch.int32),

@@ -83,6 +83,15 @@ def test_request_count_bound_checked_on_the_host():
     assert goodput(M) == ctr.CTR_OK and goodput(M + 1) == ctr.CTR_EINVAL
     tcfg = ctr.trace_cfg_struct(W.TraceCfg())
     assert L.ctr_gen_trace(ctypes.byref(tcfg), 1, 0, M + 1, ctr.CtrRequests(), None) == ctr.CTR_EINVAL
+    # the standalone scorer and its traffic probe: at most CTR_SCORE_MAX_REQ requests
+    S = ctr.CTR_SCORE_MAX_REQ
+    assert S == 1 << 40
+    cv = (ctypes.c_float * ctr.CTR_SCORE_N_CONST)(*W.SCORE_CONSTS)
+    buf = ctypes.create_string_buffer(64)
+    ptr = ctypes.cast(ctypes.addressof(buf) + (-ctypes.addressof(buf)) % 16, ctypes.c_void_p)
+    for n in (S + 4, (1 << 63) - 4):
+        assert L.ctr_score_batch(ptr, ptr, ptr, n, ptr, ptr, ptr, 4, cv, ptr, ptr, None, None) == ctr.CTR_EINVAL
+        assert L.ctr_score_stream_probe(ptr, ptr, ptr, n, ptr, ptr, None) == ctr.CTR_EINVAL
 
 
 def test_struct_layout_matches_header(tmp_path):
