@@ -56,6 +56,39 @@ def test_goodput_adversarial_times(orc):
             assert (met[r], p99[r]) == orc.goodput(sc, row, tf[r], td[r]), (N, r)
 
 
+@pytest.mark.parametrize("crowd", [1, 511, 512, 513, 3000])
+def test_goodput_crowded_p99_bin(orc, crowd):
+    """The P99's rank falls among `crowd` requests whose TTFTs share one
+    logarithmic bin: up to 512 of them are counted out exactly in shared
+    memory, more go to the radix select; TTFTs at 0 and 2^32 - 1 (the ends of
+    the binned range) and a row with one TTFT of 2^32 (outside it) ride along."""
+    ctr = need_gpu()
+    rng = np.random.default_rng(crowd)
+    R, below = 3, 3500
+    above = max(1, (crowd + below) // 99 - crowd // 3)
+    N = below + crowd + above
+    rank = (99 * N + 99) // 100 - 1
+    ttft = np.concatenate([rng.integers(0, 1000, below), 10**6 + rng.integers(0, 2000, crowd),
+                           rng.integers(10**9, 2**32, above)])
+    ttft[0], ttft[-1] = 0, 2**32 - 1
+    srt = np.sort(ttft)
+    if crowd > 1:
+        assert 10**6 <= srt[rank] < 10**6 + 2000, "the P99 must lie in the crowded bin"
+    tf = np.empty((R, N), dtype=np.int64)
+    arr = np.sort(rng.integers(0, 10**7, (R, N)), axis=1)
+    for r in range(R):
+        tf[r] = arr[r] + rng.permutation(ttft)
+    tf[2, N // 2] = arr[2, N // 2] + 2**32  # outside [0, 2^32): the whole row takes the radix select
+    trh = {"arrival_us": arr, "prompt_len": np.ones((R, N)), "true_out": rng.integers(1, 4, (R, N)),
+           "pred_out": np.ones((R, N)), "slo_class": rng.integers(0, 4, (R, N))}
+    td = tf + rng.integers(0, 20, (R, N))
+    sc = W.SimCfg(n_classes=4, ttft_slo_us=(10**3, 10**6, 10**9, 10**12), tpot_slo_us=(1, 5, 10, 10**9))
+    met, p99 = _goodput(ctr, sc, to_dev(trh), R, 1, N, torch.from_numpy(tf).cuda(), torch.from_numpy(td).cuda())
+    for r in range(R):
+        row = {k: v[r] for k, v in trh.items()}
+        assert (met[r], p99[r]) == orc.goodput(sc, row, tf[r], td[r]), (crowd, r)
+
+
 def test_goodput_empty(orc):
     ctr = need_gpu()
     tr = ctr.empty_requests(2, 0, "cuda")
