@@ -24,8 +24,9 @@
 // an arrival's own time are processed before it is routed).
 //
 // Per-lane structures live in the workspace slot of the warp, each lane's
-// entries contiguous (a heap's levels then share cache lines, and a sift-down
-// reads both children in one access): a min-heap of
+// entries contiguous (a heap's top levels then share cache lines; the heaps
+// are 4-ary, so a sift-down reads a node's four children as two 16-byte words
+// and a heap of n keys is about log4 n levels deep): a min-heap of
 // pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
 // lanes use the same region as their in-flight ring of prefill end times,
 // packed with the prompt length as end << 21 | p), a min-heap of active
@@ -111,24 +112,27 @@ __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
     return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
-// Entries per lane of a heap region holding up to cap keys: the heap is 1-based
-// (h[1] the root, h[0] unused) and a sift-down reads the children 2i and 2i + 1
-// as one 16-byte word, so the region has cap + 2 entries rounded up to even.
-__host__ __device__ __forceinline__ int64_t heap_stride(int64_t cap) { return (cap + 3) & ~int64_t(1); }
+// Entries per lane of a heap region holding up to cap keys.  The heaps are
+// 4-ary: node j (0-based) sits at position j + 3, so its children 4j + 1 ..
+// 4j + 4 sit at positions 4j + 4 .. 4j + 7, a 32-byte aligned block read as
+// two 16-byte words; the region has cap + 3 entries rounded up to 4.
+__host__ __device__ __forceinline__ int64_t heap_stride(int64_t cap) { return (cap + 6) & ~int64_t(3); }
 
-// min-heap of unique 64-bit keys in h[1..n]; each lane's heap is contiguous
+constexpr int kHeapRoot = 3;
+
+// min-heap of unique 64-bit keys; each lane's heap is contiguous
 __device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
 {
-    int i = ++n;
-    while (i > 1) {
-        const int parent = i >> 1;
+    int i = kHeapRoot + n++;
+    while (i > kHeapRoot) {
+        const int parent = (i >> 2) + 2;
         const uint64_t pv = h[parent];
         if (pv < key) break;
         h[i] = pv;
         i = parent;
     }
     h[i] = key;
-    if (i == 1) top = key;
+    if (i == kHeapRoot) top = key;
 }
 
 __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
@@ -138,25 +142,35 @@ __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
         top = kEmpty;
         return;
     }
-    const uint64_t last = h[m];
-    const int sz = m - 1;
-    int i = 1;
+    const int lastp = kHeapRoot + m - 1;
+    const uint64_t last = h[lastp];
+    const int endp = lastp - 1;  // position of the last key that stays
+    int i = kHeapRoot;
     for (;;) {
-        const int c = 2 * i;
-        if (c > sz) break;
-        const ulonglong2 ch = *reinterpret_cast<const ulonglong2*>(h + c);  // c even: a 16-byte word
-        uint64_t cv = ch.x;
+        const int c = (i - 2) << 2;  // first child
+        if (c > endp) break;
+        const ulonglong2 c01 = *reinterpret_cast<const ulonglong2*>(h + c);
+        const ulonglong2 c23 = *reinterpret_cast<const ulonglong2*>(h + c + 2);
+        uint64_t cv = c01.x;
         int ci = c;
-        if (c < sz && ch.y < cv) {
-            cv = ch.y;
+        if (c + 1 <= endp && c01.y < cv) {
+            cv = c01.y;
             ci = c + 1;
+        }
+        if (c + 2 <= endp && c23.x < cv) {
+            cv = c23.x;
+            ci = c + 2;
+        }
+        if (c + 3 <= endp && c23.y < cv) {
+            cv = c23.y;
+            ci = c + 3;
         }
         if (last < cv) break;
         h[i] = cv;
         i = ci;
     }
     h[i] = last;
-    top = h[1];
+    top = h[kHeapRoot];
 }
 
 // argmin over the lanes of 64-bit values (ties -> lowest lane)
@@ -404,7 +418,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
     if (slot >= P.n_slots) return;
     unsigned char* sb = P.ws + slot * P.slot_bytes;
     const int64_t pr_stride = heap_stride(P.cap_pr);
-    uint64_t* pend = reinterpret_cast<uint64_t*>(sb) + lane * pr_stride;  // decode lanes: 1-based heap
+    uint64_t* pend = reinterpret_cast<uint64_t*>(sb) + lane * pr_stride;  // decode lanes: 4-ary heap
     int64_t* ring = reinterpret_cast<int64_t*>(sb) + lane * pr_stride;    // prefill lanes: ring from 0
     uint64_t* act = reinterpret_cast<uint64_t*>(sb + P.off_act) + lane * heap_stride(P.cap_act);
     uint32_t* wait = reinterpret_cast<uint32_t*>(sb + P.off_wait) + lane * P.cap_wait;
