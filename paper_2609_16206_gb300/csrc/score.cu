@@ -43,9 +43,11 @@ struct __align__(16) Smem {
     int valid_tmp[4][kMaxInst];
     int pareto[4][kMaxInst];
     float seg_lo[4][kMaxInst];
-    float4 seg_e[4][kMaxInst];  // per segment: sigma w_s kappa, sigma w_s, sigma BK + WQA, index (as bits)
-    float4 brk[4][2];  // breakpoints 1..7 of each class (seg_lo[s][1..7]), +inf past the last
-    int nseg[4];
+    // per segment: sigma w_s kappa tau_dec rho, sigma w_s, sigma BK + WQA, index (as bits); row 4 holds
+    // the one entry of the invalid classes (slo_class >= 4): (0, 0, NaN, -1)
+    float4 seg_e[5][kMaxInst];
+    float4 brk[5][2];  // breakpoints 1..7 of each class (seg_lo[s][1..7]), +inf past the last; row 4 all +inf
+    int nseg[5];
     unsigned long long bar;
 };
 
@@ -78,25 +80,19 @@ __device__ __forceinline__ void line_of(const Smem& sm, const ScoreParams& P, in
     m = sig * P.c[1] * P.c[6] * P.c[3] * sm.kap[d];
 }
 
-// The request-only part of the cost: own = G + H * kappa_d with
-// G = tau_pre0 + tau_pre p + tau_dec o_hat (1 + rho (p + o_hat) / C) and H = tau_dec rho o_hat,
-// so cost = sigma_s (BK_d + w_s (G + H kappa_d)) + WQA_d.
-struct ReqTerms {
-    float g, h;
-};
-
-__device__ __forceinline__ ReqTerms req_terms(const ScoreParams& P, float p, float oh)
+// The request-only part of the cost: own = G + H kappa_d with
+// G = tau_pre0 + tau_pre p + o_hat (tau_dec + tau_dec rho / C (p + o_hat)) and H = tau_dec rho o_hat,
+// so cost = sigma_s (BK_d + w_s (G + H kappa_d)) + WQA_d.  The constant tau_dec rho / C is
+// folded once per thread (kg) and tau_dec rho into the segment entries.
+__device__ __forceinline__ float req_g(const ScoreParams& P, float kg, float p, float oh)
 {
-    const float toh = P.c[6] * oh;                                   // tau_dec o_hat
-    const float press_req = (p + oh) * P.c[8];                       // (p + o_hat) / C
-    const float g = fmaf(toh, fmaf(P.c[3], press_req, 1.0f), fmaf(P.c[5], p, P.c[4]));
-    return ReqTerms{g, toh * P.c[3]};
+    return fmaf(oh, fmaf(kg, p + oh, P.c[6]), fmaf(P.c[5], p, P.c[4]));
 }
 
-// The full cost at the segment's instance, e = (sigma_s w_s kappa_d, sigma_s w_s,
-// sigma_s BK_d + WQA_d, d): sigma_s w_s kappa_d H + sigma_s w_s G + sigma_s BK_d + WQA_d,
-// every term non-negative, each path at most 7 roundings of 2^-24.
-__device__ __forceinline__ float cost_at(ReqTerms r, float4 e) { return fmaf(e.x, r.h, fmaf(e.y, r.g, e.z)); }
+// The full cost at the segment's instance, e = (sigma_s w_s tau_dec rho kappa_d, sigma_s w_s,
+// sigma_s BK_d + WQA_d, d): e.x o_hat + e.y G + e.z, every term non-negative, each path
+// at most 9 roundings of 2^-24.
+__device__ __forceinline__ float cost_at(float g, float oh, float4 e) { return fmaf(e.x, oh, fmaf(e.y, g, e.z)); }
 
 // the segment entry of instance d in class s
 __device__ __forceinline__ float4 seg_entry(const Smem& sm, const ScoreParams& P, int s, int d)
@@ -105,20 +101,17 @@ __device__ __forceinline__ float4 seg_entry(const Smem& sm, const ScoreParams& P
     const float sig = P.c[9 + s];
     const float sws = sig * P.c[1];
     const float bk = P.c[0] * fmaf(P.c[5], sm.q[d], P.c[7] * A);
-    return make_float4(sws * sm.kap[d], sws, fmaf(sig, bk, P.c[2] * A), __int_as_float(d));
+    return make_float4(sws * sm.kap[d] * P.c[6] * P.c[3], sws, fmaf(sig, bk, P.c[2] * A), __int_as_float(d));
 }
 
 // kB = 4 or 8: every class has at most kB + 1 segments (block-uniform), and the
 // segment is the count of its padded breakpoints <= o_hat; kB = 0: binary search
+// (an invalid class reads row 4: no breakpoints, one entry (0, 0, NaN, -1))
 template <int kB>
-__device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, float p, float oh, uint32_t s,
-                                          int& arg, float& cost)
+__device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, float kg, float p, float oh,
+                                          uint32_t s, int& arg, float& cost)
 {
-    if (s >= 4) {
-        arg = -1;
-        cost = __int_as_float(0x7fc00000);
-        return;
-    }
+    s = s < 4u ? s : 4u;
     int seg;
     if (kB > 0) {  // segments start at 0 and at the sorted breakpoints: count those <= o_hat
         const float4 b0 = sm.brk[s][0];
@@ -138,7 +131,7 @@ __device__ __forceinline__ void score_one(const Smem& sm, const ScoreParams& P, 
     }
     const float4 e = sm.seg_e[s][seg];
     arg = __float_as_int(e.w);
-    cost = cost_at(req_terms(P, p, oh), e);
+    cost = cost_at(req_g(P, kg, p, oh), oh, e);
 }
 
 // (intercept, slope, index) lexicographic order of envelope lines
@@ -155,31 +148,32 @@ __device__ __forceinline__ uint32_t fkey(float x)
     return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-// Lexicographic (x, m, j) minimum over the warp of each lane's candidate,
-// returned to every lane as the winning index j (-1 when no lane has one):
-// three redux.sync minimum reductions, on the key of x, then on the key of m
-// among the lanes holding that x, then on j among those holding both.
-__device__ __forceinline__ int warp_lexmin(bool has, float x, float m, int j)
+// The warp's least (x, j) over each lane's candidate, returned to every lane as
+// the winning index j (-1 when no lane has one): a redux.sync minimum on the
+// key of x, then one on j among the lanes holding that x.
+__device__ __forceinline__ int warp_argmin_x(bool has, float x, int j)
 {
     const uint32_t kx = has ? fkey(x) : 0xffffffffu;
     const uint32_t mx = __reduce_min_sync(0xffffffffu, kx);
-    const bool at_x = has && kx == mx;
-    const uint32_t km = at_x ? fkey(m) : 0xffffffffu;
-    const uint32_t mm = __reduce_min_sync(0xffffffffu, km);
-    const uint32_t kj = at_x && km == mm ? (uint32_t)j : 0xffffffffu;
+    const uint32_t kj = has && kx == mx ? (uint32_t)j : 0xffffffffu;
     return (int)__reduce_min_sync(0xffffffffu, kj);
 }
 
 // Lower envelope of one class's lines over o_hat >= 0 with one warp, for up to
-// 64 lines (two per lane), by gift wrapping: the first segment's line is the
-// least (intercept, slope, index); from the current line the next one is,
-// among the lines of smaller slope, the one whose crossing with it comes first
-// (ties: smaller slope, then lower index), and the crossing is that segment's
-// left end.  Each step lowers the slope, so the loop ends within n_inst steps,
-// one warp minimum each (a handful for the states seen in practice: the
-// envelope of n random lines has O(log n) segments).  A lane's two lines are
-// compared first, then the warp takes the minimum with two redux.sync
-// reductions and a ballot.  Left ends are kept non-decreasing against
+// 64 lines (two per lane), by gift wrapping: the first segment's line has the
+// least intercept; from the current line the next one is, among the lines of
+// smaller slope, the one whose crossing with it comes first, and the crossing
+// is that segment's left end.  Each step lowers the slope, so the loop ends
+// within n_inst steps, one warp minimum each (a handful for the states seen in
+// practice: the envelope of n random lines has O(log n) segments).  Ties need
+// no slope rule: of two lines meeting the current one at the same point, the
+// steeper one taken first meets the other there again at the next step, which
+// leaves it a segment of zero length (a crossing a rounding step off leaves a
+// sliver where the two costs agree to rounding).  A lane's two lines are
+// compared first (least crossing, then smaller slope), then the warp takes
+// the least (crossing, index) with two redux.sync reductions.  Crossings use
+// the fast reciprocal divide (a few ulp, which moves a breakpoint only among
+// near-equal costs).  Left ends are kept non-decreasing against
 // rounding.  Segment t stays in lane t % 32, slot t / 32, until the warp writes
 // the segment arrays and the padded breakpoints.
 __device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst, int lane)
@@ -199,10 +193,10 @@ __device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst,
         // every comparison below a total order and the warp's decisions uniform
         live[r] = fabsf(a[r]) < inf && fabsf(m[r]) < inf;
     }
-    // the lane's least line, then the warp's: (intercept, slope, index)
+    // the lane's least line (intercept, slope, index), then the warp's (intercept, index)
     int r0 = live[0] ? 0 : 1;
     if (live[0] && live[1] && line_less(a[1], m[1], lane + 32, a[0], m[0], lane)) r0 = 1;
-    int ci = warp_lexmin(live[0] || live[1], r0 ? a[1] : a[0], r0 ? m[1] : m[0], lane + 32 * r0);
+    int ci = warp_argmin_x(live[0] || live[1], r0 ? a[1] : a[0], lane + 32 * r0);
     bool more = ci >= 0;
     if (!more) ci = 0;  // no finite line at all (outside the input contract): line 0
     float ca = __shfl_sync(0xffffffffu, ci >= 32 ? a[1] : a[0], ci & 31);
@@ -212,26 +206,19 @@ __device__ void warp_envelope(Smem& sm, const ScoreParams& P, int s, int n_inst,
     float x_cur = 0.0f;
     int nseg = 1;
     while (more && nseg < n_inst) {
-        // the lane's first crossing among its lines of smaller slope (x, slope, index)
-        bool has = false;
-        float bx = inf, bm = inf;
-        int br = 0;
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            if (live[r] && m[r] < cm) {
-                const float x = (a[r] - ca) / (cm - m[r]);
-                if (x == x && (!has || x < bx || (x == bx && m[r] < bm))) {  // slot 0 (lower index) on full ties
-                    has = true;
-                    bx = x;
-                    bm = m[r];
-                    br = r;
-                }
-            }
-        }
-        const int bi = warp_lexmin(has, bx, bm, lane + 32 * br);  // the warp's first crossing
+        // the lane's first crossing among its lines of smaller slope (x, slope, index),
+        // branch-free: both crossings, then selects
+        const float d0 = cm - m[0], d1 = cm - m[1];
+        const float x0 = __fdividef(a[0] - ca, d0), x1 = __fdividef(a[1] - ca, d1);
+        const bool c0 = live[0] && m[0] < cm && x0 == x0;
+        const bool c1 = live[1] && m[1] < cm && x1 == x1;
+        const bool p1 = c1 && (!c0 || x1 < x0 || (x1 == x0 && m[1] < m[0]));  // slot 0 (lower index) on full ties
+        const bool has = c0 || c1;
+        const float bx = p1 ? x1 : x0, bm = p1 ? m[1] : m[0], ba = p1 ? a[1] : a[0];
+        const int bi = warp_argmin_x(has, bx, lane + 32 * (int)p1);  // the warp's first crossing
         if (bi < 0) break;  // warp-uniform: no line of smaller slope is left
         const int wl = bi & 31;
-        ca = __shfl_sync(0xffffffffu, bi >= 32 ? a[1] : a[0], wl);
+        ca = __shfl_sync(0xffffffffu, ba, wl);
         cm = __shfl_sync(0xffffffffu, bm, wl);
         x_cur = fmaxf(__shfl_sync(0xffffffffu, bx, wl), x_cur);
         if (lane == (nseg & 31)) {
@@ -305,6 +292,7 @@ __device__ __forceinline__ void pipe_score(ReqPipe& q, const Smem& sm, const Sco
     const uint32_t* c4 = reinterpret_cast<const uint32_t*>(P.cls);
     int4* a4 = reinterpret_cast<int4*>(P.argmin);
     float4* f4 = reinterpret_cast<float4*>(P.cost);
+    const float kg = P.c[6] * P.c[3] * P.c[8];
     while (q.has) {
         const int64_t vf = q.v + 2 * kThreads;
         const bool hf = vf < q.end;
@@ -317,10 +305,10 @@ __device__ __forceinline__ void pipe_score(ReqPipe& q, const Smem& sm, const Sco
         }
         int4 ai;
         float4 fc;
-        score_one<kB>(sm, P, q.pv.x, q.ov.x, q.cv & 0xFFu, ai.x, fc.x);
-        score_one<kB>(sm, P, q.pv.y, q.ov.y, (q.cv >> 8) & 0xFFu, ai.y, fc.y);
-        score_one<kB>(sm, P, q.pv.z, q.ov.z, (q.cv >> 16) & 0xFFu, ai.z, fc.z);
-        score_one<kB>(sm, P, q.pv.w, q.ov.w, q.cv >> 24, ai.w, fc.w);
+        score_one<kB>(sm, P, kg, q.pv.x, q.ov.x, q.cv & 0xFFu, ai.x, fc.x);
+        score_one<kB>(sm, P, kg, q.pv.y, q.ov.y, (q.cv >> 8) & 0xFFu, ai.y, fc.y);
+        score_one<kB>(sm, P, kg, q.pv.z, q.ov.z, (q.cv >> 16) & 0xFFu, ai.z, fc.z);
+        score_one<kB>(sm, P, kg, q.pv.w, q.ov.w, q.cv >> 24, ai.w, fc.w);
         __stcs(a4 + q.v, ai);
         __stcs(f4 + q.v, fc);
         q.v += kThreads;
@@ -342,6 +330,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
     Smem& sm = *reinterpret_cast<Smem*>(smem_raw);
     const int tid = threadIdx.x;
     const int n_inst = P.n_inst;
+    if (tid == kThreads - 1) {  // row 4: the invalid classes (visible after the first barrier)
+        const float inf = __int_as_float(0x7f800000);
+        sm.brk[4][0] = sm.brk[4][1] = make_float4(inf, inf, inf, inf);
+        sm.seg_e[4][0] = make_float4(0.0f, 0.0f, __int_as_float(0x7fc00000), __int_as_float(-1));
+        sm.nseg[4] = 1;
+    }
 
     // ---- stage the instance state first: it heads the critical path (state -> envelopes -> scoring), so
     // its TMA bulk copy is issued before the request prefetch (plain loads when unaligned)
@@ -527,7 +521,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
             const int64_t i = (nv << 2) + tid;
             int ai;
             float fc;
-            score_one<0>(sm, P, P.p[i], P.oh[i], P.cls[i], ai, fc);
+            score_one<0>(sm, P, P.c[6] * P.c[3] * P.c[8], P.p[i], P.oh[i], P.cls[i], ai, fc);
             P.argmin[i] = ai;
             P.cost[i] = fc;
         }
@@ -535,7 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const ScoreParams P)
         for (int64_t i = (int64_t)blockIdx.x * kThreads + tid; i < P.n; i += (int64_t)gridDim.x * kThreads) {
             int ai;
             float fc;
-            score_one<0>(sm, P, P.p[i], P.oh[i], P.cls[i], ai, fc);
+            score_one<0>(sm, P, P.c[6] * P.c[3] * P.c[8], P.p[i], P.oh[i], P.cls[i], ai, fc);
             P.argmin[i] = ai;
             P.cost[i] = fc;
         }
