@@ -303,28 +303,30 @@ def run_ours(args, rank, world, local_rank):
     sam = torch.empty(N_SCORE_REQ, dtype=torch.int32, device=dev)
     scost = torch.empty(N_SCORE_REQ, dtype=torch.float32, device=dev)
 
-    ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(2)] for k in ("gen", "sim", "score")}
-    times = {k: 0.0 for k in ev}
+    marks = {k: [] for k in ("gen", "sim", "score")}
 
     def step(timed: bool):
+        """One pass of the hot path: trace generation, simulation (then each row's checksum and goodput in
+        one pass over the outputs) and the scorer; with `timed`, CUDA events around each kernel, read after
+        the timed region (no host synchronisation between steps)."""
+        e = {k: [torch.cuda.Event(enable_timing=True) for _ in range(2)] for k in marks} if timed else None
+
         def mark(name, i):
             if timed:
-                ev[name][i].record(stream)
+                e[name][i].record(stream)
         mark("gen", 0)
         ctr.ctr_gen_trace(wl.trace, R, offset, N, tr, stream=stream)
         mark("gen", 1)
-        mark("sim", 0)  # simulation, then each row's checksum and goodput in one pass over the outputs
+        mark("sim", 0)
         ctr.ctr_simulate(wl.sim, [W.CALIBRATED], pols, tr, R, N, tf, td, rhash, rstat, ws, met_count=met,
                          p99_ttft_us=p99, stream=stream)
         mark("sim", 1)
         mark("score", 0)
         ctr.ctr_score_batch(sp, soh, scls, sQ, sA, skap, W.SCORE_CONSTS, sam, scost, stream=stream)
         mark("score", 1)
-
-    def accumulate():
-        torch.cuda.synchronize()
-        for k, (a, b) in ev.items():
-            times[k] += a.elapsed_time(b)
+        if timed:
+            for k in e:
+                marks[k].append(e[k])
 
     for _ in range(args.warmup):
         step(False)
@@ -342,9 +344,9 @@ def run_ours(args, rank, world, local_rank):
     t0.record(stream)
     for _ in range(args.steps):
         step(True)
-        accumulate()
     t1.record(stream)
     torch.cuda.synchronize()
+    times = {k: sum(a.elapsed_time(z) for a, z in v) for k, v in marks.items()}
     if world > 1:
         torch.distributed.barrier()
     clk = clocks.stop() if rank == 0 else None
