@@ -606,17 +606,17 @@ def run_ours(args, rank, world, local_rank):
 # per routed request, keyed by a hash of the simulator's code: a stale entry
 # (the kernel changed since the counters were taken) reports null.
 SIM_SLICE_COUNTERS: dict = {
-    "8d95302a87f8aff8": {"warp_inst_per_routed": 34196262584 / 81_920_000,
-                         "thread_inst_per_warp_inst": 281902365249 / 34196262584,
-                         "dram_bytes_per_routed": (2382569216 + 1571453440) / 81_920_000,
+    "7fec69fccc56e65d": {"warp_inst_per_routed": 34090777159 / 81_920_000,
+                         "thread_inst_per_warp_inst": 280855382989 / 34090777159,
+                         "dram_bytes_per_routed": (2383783168 + 1564177152) / 81_920_000,
                          "slice": "ncu on one launch of 1,024 replicas x 20,000 requests x 4 policies "
-                                  "(81.92 M routed requests): 3.420e10 warp-instructions, 2.819e11 thread-"
-                                  "instructions, 2.383 GB DRAM read + 1.571 GB written"},
+                                  "(81.92 M routed requests): 3.409e10 warp-instructions, 2.809e11 thread-"
+                                  "instructions, 2.384 GB DRAM read + 1.564 GB written"},
 }
 
 # DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.
 SCORE_DRAM_PER_LAUNCH: dict = {
-    "55623de89a963cd4": {"read": 9480704.0, "write": 0.0},
+    "86ed7794a9408ef3": {"read": 9485312.0, "write": 0.0},
 }
 
 

@@ -25,8 +25,8 @@
 //
 // Per-lane structures live in the workspace slot of the warp, each lane's
 // entries contiguous (a heap's top levels then share cache lines; the heaps
-// are 4-ary, so a sift-down reads a node's four children as two 16-byte words
-// and a heap of n keys is about log4 n levels deep): a min-heap of
+// are 4-ary, a node's four children two 16-byte words and a heap of n keys
+// about log4 n levels deep, except with batched prefill: see HeapShape): a min-heap of
 // pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
 // lanes use the same region as their in-flight ring of prefill end times,
 // packed with the prompt length as end << 21 | p), a min-heap of active
@@ -112,65 +112,81 @@ __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
     return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
-// Entries per lane of a heap region holding up to cap keys.  The heaps are
-// 4-ary: node j (0-based) sits at position j + 3, so its children 4j + 1 ..
-// 4j + 4 sit at positions 4j + 4 .. 4j + 7, a 32-byte aligned block read as
-// two 16-byte words; the region has cap + 3 entries rounded up to 4.
+// Entries per lane of a heap region holding up to cap keys, for either arity below:
+// cap + 3 entries rounded up to 4 (a 32-byte multiple).
 __host__ __device__ __forceinline__ int64_t heap_stride(int64_t cap) { return (cap + 6) & ~int64_t(3); }
 
-constexpr int kHeapRoot = 3;
+// Min-heaps of unique 64-bit keys, each lane's heap contiguous.  kArity 4: node j
+// (0-based) at position j + 3, its children 4j + 1 .. 4j + 4 at positions
+// 4j + 4 .. 4j + 7, one 32-byte aligned block read as two 16-byte words, about
+// log4 n levels: fewer dependent loads per pop, more compares per level.  kArity
+// 2: 1-based, children 2i and 2i + 1 one 16-byte word.  The kernel takes 4 for
+// long decode batches (the replica sweep's and the large pool's: -2 % and -6 %
+// there) and 2 with batched prefill, whose short-output document workload keeps
+// the batches small (4-ary is 6 % slower there).
+template <int kArity>
+struct HeapShape {
+    static constexpr int kRoot = kArity == 4 ? 3 : 1;
+    __device__ static __forceinline__ int parent(int i) { return kArity == 4 ? (i >> 2) + 2 : i >> 1; }
+    __device__ static __forceinline__ int first_child(int i) { return kArity == 4 ? (i - 2) << 2 : i << 1; }
+};
 
-// min-heap of unique 64-bit keys; each lane's heap is contiguous
+template <int kArity>
 __device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
 {
-    int i = kHeapRoot + n++;
-    while (i > kHeapRoot) {
-        const int parent = (i >> 2) + 2;
+    using S = HeapShape<kArity>;
+    int i = S::kRoot + n++;
+    while (i > S::kRoot) {
+        const int parent = S::parent(i);
         const uint64_t pv = h[parent];
         if (pv < key) break;
         h[i] = pv;
         i = parent;
     }
     h[i] = key;
-    if (i == kHeapRoot) top = key;
+    if (i == S::kRoot) top = key;
 }
 
+template <int kArity>
 __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
 {
+    using S = HeapShape<kArity>;
     const int m = n--;  // the last key moves into the hole left at the root
     if (m == 1) {
         top = kEmpty;
         return;
     }
-    const int lastp = kHeapRoot + m - 1;
+    const int lastp = S::kRoot + m - 1;
     const uint64_t last = h[lastp];
     const int endp = lastp - 1;  // position of the last key that stays
-    int i = kHeapRoot;
+    int i = S::kRoot;
     for (;;) {
-        const int c = (i - 2) << 2;  // first child
+        const int c = S::first_child(i);
         if (c > endp) break;
         const ulonglong2 c01 = *reinterpret_cast<const ulonglong2*>(h + c);
-        const ulonglong2 c23 = *reinterpret_cast<const ulonglong2*>(h + c + 2);
         uint64_t cv = c01.x;
         int ci = c;
         if (c + 1 <= endp && c01.y < cv) {
             cv = c01.y;
             ci = c + 1;
         }
-        if (c + 2 <= endp && c23.x < cv) {
-            cv = c23.x;
-            ci = c + 2;
-        }
-        if (c + 3 <= endp && c23.y < cv) {
-            cv = c23.y;
-            ci = c + 3;
+        if (kArity == 4) {
+            const ulonglong2 c23 = *reinterpret_cast<const ulonglong2*>(h + c + 2);
+            if (c + 2 <= endp && c23.x < cv) {
+                cv = c23.x;
+                ci = c + 2;
+            }
+            if (c + 3 <= endp && c23.y < cv) {
+                cv = c23.y;
+                ci = c + 3;
+            }
         }
         if (last < cv) break;
         h[i] = cv;
         i = ci;
     }
     h[i] = last;
-    top = h[kHeapRoot];
+    top = h[S::kRoot];
 }
 
 // argmin over the lanes of 64-bit values (ties -> lowest lane)
@@ -198,11 +214,12 @@ struct Decode {
 
 // Move every pending request whose KV is ready by t into the waiting FIFO, in
 // (time, index) order; the FIFO's size is checked after each insertion.
+template <int kArity>
 __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams& P, uint64_t* pend, uint32_t* wait)
 {
     while (s.pend_n > 0 && (int64_t)(s.pend_top >> kKeyBits) <= t) {
         const uint32_t k = (uint32_t)(s.pend_top & kKeyMask);
-        heap_pop(pend, s.pend_n, s.pend_top);
+        heap_pop<kArity>(pend, s.pend_n, s.pend_top);
         if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
         int pos = s.w_head + s.w_n;
         if (pos >= P.cap_wait) pos -= P.cap_wait;
@@ -218,7 +235,7 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
 // FIFO has overflowed.  kSnap: when tsnap >= 0, also record in kv_snap the
 // resident KV as it is after every event at times <= tsnap (an occupancy
 // poll; tsnap <= T), then set tsnap to -1.
-template <bool kSnap>
+template <bool kSnap, int kArity>
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
                                               uint32_t* wait, int64_t tb, int64_t ob, int64_t& tsnap, int64_t& kv_snap,
                                               bool sum_is_o_hat)
@@ -294,7 +311,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.stepping = false;
             while (s.n_act > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
                 const int64_t k = (int64_t)(s.act_top & kKeyMask);
-                heap_pop(act, s.n_act, s.act_top);
+                heap_pop<kArity>(act, s.n_act, s.act_top);
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
                 s.q -= 1;
@@ -305,7 +322,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             }
         }
         // (2) every request KV-ready by now joins the waiting FIFO in (time, index) order
-        const int rc = flush_ready(s, tev, P, pend, wait);
+        const int rc = flush_ready<kArity>(s, tev, P, pend, wait);
         if (rc != CTR_OK) return rc;
         // (3) not mid-step: strict FCFS admission while the reservation fits, then start a step
         if (!s.stepping) {
@@ -321,7 +338,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 s.w_n -= 1;
                 s.kv_rsv += (int32_t)(pk + ok);
                 s.kv_res += (int32_t)pk;
-                heap_push(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
+                heap_push<kArity>(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
                 admitted += 1;
             }
             if (s.n_act > 0) {
@@ -409,6 +426,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
 {
     constexpr bool kSig = kMode >= 1;  // the proxy's signals: ledger backlog, polled occupancy
     constexpr bool kBat = kMode == 2;  // batched prefill
+    constexpr int kArity = kBat ? 2 : 4;  // heap arity (see HeapShape)
     constexpr int kRowsPerWarp = 32 / G;
     const int lane = threadIdx.x & 31;
     const int grp = lane / G;
@@ -531,7 +549,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 if (s.pend_n == P.cap_pend_store) {
                                     err = CTR_EOVERFLOW;  // the waiting FIFO has overflowed
                                 } else {
-                                    heap_push(pend, s.pend_n, s.pend_top,
+                                    heap_push<kArity>(pend, s.pend_n, s.pend_top,
                                               ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift));
                                 }
                             }
@@ -576,7 +594,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 last_poll = tp;
                             }
                         }
-                        if (err == CTR_OK) err = decode_advance<kSig>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen, sum_is_o_hat);
+                        if (err == CTR_OK) err = decode_advance<kSig, kArity>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen, sum_is_o_hat);
                     } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
                         while (ring_n > 0 && ring_front <= (uint64_t)thr) {
@@ -736,12 +754,12 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 if (live && gl == P.n_pre + id && ready < kTimeLimit) {
                     // requests routed here whose KV is not ready yet, exactly: first move
                     // those already ready (kept in the heap until the step end) if it matters
-                    if (s.q - s.w_n - s.n_act >= P.cap_pend) err = flush_ready(s, T, P, pend, wait);
+                    if (s.q - s.w_n - s.n_act >= P.cap_pend) err = flush_ready<kArity>(s, T, P, pend, wait);
                     if (err != CTR_OK || s.q - s.w_n - s.n_act == P.cap_pend ||
                         (ready >= 0 && s.pend_n == P.cap_pend_store)) {
                         err = CTR_EOVERFLOW;
                     } else {
-                        if (ready >= 0) heap_push(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
+                        if (ready >= 0) heap_push<kArity>(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
                         s.q += 1;
                         s.sum += sum_is_o_hat ? ohk : ok;
                     }
@@ -766,7 +784,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         }
         if (live && is_dec) {
             int64_t no_snap = -1;
-            err = decode_advance<false>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, sum_is_o_hat);
+            err = decode_advance<false, kArity>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, sum_is_o_hat);
         }
 
 #pragma unroll
