@@ -2,18 +2,22 @@
 // the count of requests meeting both SLOs of their class (sec. IV-B targets,
 // Table 2 goodput) and the exact nearest-rank P99 TTFT (Table 2 column).
 //
-// One block per row.  Pass 0 reads the row once: the met count, and, when the
-// row fits in shared memory (kStage) and every TTFT lies in [0, 2^32), a
-// histogram of the TTFTs over logarithmic bins (64 per octave, monotone in the
-// TTFT) with each request's bin kept in shared memory.  A block scan finds the
-// bin holding the P99's rank; the requests of that bin (a few dozen in
+// One block per unit of up to kRows rows of one replica, which share the
+// replica's trace and request indices.  Pass 0 reads the unit once: per
+// request the trace's arrival, output length and class, then each row's
+// t_first and t_done; per row the met count and, when the rows fit in shared
+// memory (kStage) and every TTFT lies in [0, 2^32), a histogram of the TTFTs
+// over logarithmic bins (64 per octave, monotone in the TTFT) with each
+// request's bin kept in shared memory.  For each row a block scan then finds
+// the bin holding the P99's rank; the requests of that bin (a few dozen in
 // practice) are gathered, their exact TTFTs read back, and the value of the
-// remaining rank among them counted out exactly.  A row with too many requests,
-// a TTFT outside [0, 2^32) or more than kCand requests in the P99's bin falls
-// back to a radix select over the exact TTFTs read from global memory
-// (11-bit digits, most significant first).  Called from ctr_simulate with
-// kHash, pass 0 also sums the row checksum's first-token and completion terms,
-// so the outputs are read once for both.
+// remaining rank among them counted out exactly.  A row with a TTFT outside
+// [0, 2^32), more than kCand requests in the P99's bin, or too many requests
+// to stage falls back to a radix select over the exact TTFTs read from global
+// memory (11-bit digits, most significant first).  Called from ctr_simulate
+// with kHash, pass 0 also sums each row's checksum terms of first-token and
+// completion times; the request-only half of those terms is mixed once per
+// request for the unit's rows.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -91,154 +95,210 @@ __device__ void find_rank_bin(const uint32_t* hist, int nb, int64_t rank, uint32
     __syncthreads();
 }
 
-template <bool kStage, bool kHash>
-__global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParams P)
-{
-    __shared__ uint32_t hist[kLogBins];
-    __shared__ int64_t red64[kThreads / 32];
-    __shared__ uint32_t wsum[kThreads / 32];
-    __shared__ uint32_t pick[2];
-    __shared__ uint32_t n_cand;
-    __shared__ int32_t cand_k[kCand];
-    __shared__ int64_t cand_v[kCand];
-    extern __shared__ uint16_t bin_s[];  // kStage: each request's TTFT bin
-    const int tid = threadIdx.x;
-    const int64_t n = P.n_req;
 
-    for (int64_t row = blockIdx.x; row < P.n_rows; row += gridDim.x) {
-        const int64_t tb = (row / P.rows_per_replica) * n;
-        const int64_t ob = row * n;
-        if (kStage) {
-            for (int i = tid; i < kLogBins; i += kThreads) hist[i] = 0;
-            if (tid == 0) n_cand = 0;
-            __syncthreads();
-        }
-        int32_t met = 0;
-        bool wide = false;  // some TTFT outside [0, 2^32)
-        uint64_t h = 0;     // kHash: the row's first-token and completion checksum terms
-        // 2 elements per thread per round, all loads issued before any is used
-        for (int64_t base = tid; base < n; base += (int64_t)kThreads * 2) {
-            int64_t tf[2], td[2], ta[2];
-            int32_t ov[2];
-            uint32_t cv[2];
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const int64_t k = base + (int64_t)u * kThreads;
-                if (k < n) {
-                    tf[u] = __ldg(&P.t_first[ob + k]);
-                    td[u] = __ldg(&P.t_done[ob + k]);
-                    ta[u] = __ldg(&P.trace.arrival_us[tb + k]);
-                    ov[u] = __ldg(&P.trace.true_out[tb + k]);
-                    cv[u] = __ldg(&P.trace.slo_class[tb + k]);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const int64_t k = base + (int64_t)u * kThreads;
-                if (k < n) {
-                    const int64_t ttft = tf[u] - ta[u];
-                    const int64_t o = ov[u];
-                    int c = (int)cv[u];
-                    if (c >= P.n_classes) c = P.n_classes - 1;
-                    met += ttft <= P.ttft[c] && (o == 1 || td[u] - tf[u] <= P.tpot[c] * (o - 1));
-                    const bool fits = (uint64_t)ttft < (uint64_t(1) << 32);
-                    wide |= !fits;
-                    if (kStage) {
-                        const uint32_t b = fits ? log_bin((uint32_t)ttft) : 0u;
-                        atomicAdd(&hist[b], 1u);
-                        bin_s[k] = (uint16_t)b;
-                    }
-                    if (kHash) h += hterm(k, 2, (uint64_t)tf[u]) + hterm(k, 3, (uint64_t)td[u]);
-                }
-            }
-        }
-        met = block_reduce<int32_t>(met, 0, [](int32_t a, int32_t b) { return a + b; },
-                                    reinterpret_cast<int32_t*>(red64));
-        if (kHash) {
-            h = (uint64_t)block_reduce<int64_t>((int64_t)h, 0, [](int64_t a, int64_t b) {
-                return (int64_t)((uint64_t)a + (uint64_t)b);  // sum mod 2^64
-            }, red64);
-            if (tid == 0 && P.row_status[row] == CTR_OK) P.row_hash[row] += h;  // a failed row keeps 0
-        }
-        wide = __syncthreads_or(wide) != 0;
-        if (n == 0) {
-            if (tid == 0) {
-                P.met[row] = 0;
-                P.p99[row] = -1;
-            }
-            continue;
-        }
-        const int64_t rank = (99 * n + 99) / 100 - 1;  // 0-based nearest rank
-        if (kStage && !wide) {
-            find_rank_bin(hist, kLogBins, rank, pick, wsum);
-            const uint32_t B = pick[0];
-            const int64_t r_in = rank - (int64_t)pick[1];  // rank among the bin's requests
-            for (int64_t k = tid; k < n; k += kThreads) {
-                if (bin_s[k] == B) {
-                    const uint32_t i = atomicAdd(&n_cand, 1u);
-                    if (i < (uint32_t)kCand) cand_k[i] = (int32_t)k;
-                }
-            }
-            __syncthreads();
-            const int c = (int)n_cand;
-            if (c <= kCand) {
-                for (int i = tid; i < c; i += kThreads) {
-                    const int64_t k = cand_k[i];
-                    cand_v[i] = P.t_first[ob + k] - P.trace.arrival_us[tb + k];
-                }
-                __syncthreads();
-                // the candidate whose position in (value, slot) order is the remaining rank
-                for (int i = tid; i < c; i += kThreads) {
-                    const int64_t v = cand_v[i];
-                    int64_t pos = 0;
-                    for (int j = 0; j < c; ++j) {
-                        const int64_t w = cand_v[j];
-                        pos += w < v || (w == v && j < i);
-                    }
-                    if (pos == r_in) P.p99[row] = v;
-                }
-                if (tid == 0) P.met[row] = met;
-                __syncthreads();
-                continue;
-            }
-        }
-        // ---- fallback: exact radix select over (TTFT - min) read from global memory
-        int64_t mn = INT64_MAX, mx = INT64_MIN;
+// Shared scratch of the per-row selection.
+struct SelScratch {
+    int64_t red64[kThreads / 32];
+    uint32_t wsum[kThreads / 32];
+    uint32_t pick[2];
+    uint32_t n_cand;
+    int32_t cand_k[kCand];
+    int64_t cand_v[kCand];
+};
+
+// One row's P99 TTFT (and its met count, already reduced) into P.p99 / P.met:
+// from its histogram and staged bins when `staged`, else by the radix select
+// over the TTFTs in global memory (which reuses `hist`).  Block-collective.
+__device__ void select_row(const GoodputParams& P, int64_t row, int64_t tb, int64_t n, int32_t met, bool staged,
+                           uint32_t* hist, const uint16_t* bins, SelScratch& S)
+{
+    const int tid = threadIdx.x;
+    const int64_t ob = row * n;
+    const int64_t rank = (99 * n + 99) / 100 - 1;  // 0-based nearest rank
+    if (staged) {
+        if (tid == 0) S.n_cand = 0;
+        find_rank_bin(hist, kLogBins, rank, S.pick, S.wsum);  // its barriers also publish n_cand
+        const uint32_t B = S.pick[0];
+        const int64_t r_in = rank - (int64_t)S.pick[1];  // rank among the bin's requests
         for (int64_t k = tid; k < n; k += kThreads) {
-            const int64_t t = P.t_first[ob + k] - P.trace.arrival_us[tb + k];
-            mn = t < mn ? t : mn;
-            mx = t > mx ? t : mx;
-        }
-        mn = block_reduce<int64_t>(mn, INT64_MAX, [](int64_t a, int64_t b) { return a < b ? a : b; }, red64);
-        mx = block_reduce<int64_t>(mx, INT64_MIN, [](int64_t a, int64_t b) { return a > b ? a : b; }, red64);
-        const uint64_t range = (uint64_t)mx - (uint64_t)mn;
-        int shift = range == 0 ? 0 : 64 - __clzll((long long)range);  // bits still undetermined
-        uint64_t prefix = 0;                                            // chosen high bits of (ttft - mn)
-        int64_t rk = rank;                                              // rank among the candidates
-        while (shift > 0) {
-            const int dbits = shift < kDigit ? shift : kDigit;
-            const int above = shift;  // candidates agree with prefix on bits >= above
-            shift -= dbits;
-            for (int i = tid; i < kBins; i += kThreads) hist[i] = 0;
-            __syncthreads();
-            const uint32_t dmask = (1u << dbits) - 1u;
-            for (int64_t k = tid; k < n; k += kThreads) {
-                const uint64_t v = (uint64_t)(P.t_first[ob + k] - P.trace.arrival_us[tb + k]) - (uint64_t)mn;
-                const bool match = above >= 64 || (v >> above) == (prefix >> above);
-                if (match) atomicAdd(&hist[(uint32_t)(v >> shift) & dmask], 1u);
+            if (bins[k] == B) {
+                const uint32_t i = atomicAdd(&S.n_cand, 1u);
+                if (i < (uint32_t)kCand) S.cand_k[i] = (int32_t)k;
             }
-            __syncthreads();
-            find_rank_bin(hist, kBins, rk, pick, wsum);
-            prefix |= (uint64_t)pick[0] << shift;
-            rk -= pick[1];
-            __syncthreads();
-        }
-        if (tid == 0) {
-            P.met[row] = met;
-            P.p99[row] = (int64_t)((uint64_t)mn + prefix);
         }
         __syncthreads();
+        const int c = (int)S.n_cand;
+        if (c <= kCand) {
+            for (int i = tid; i < c; i += kThreads) {
+                const int64_t k = S.cand_k[i];
+                S.cand_v[i] = P.t_first[ob + k] - P.trace.arrival_us[tb + k];
+            }
+            __syncthreads();
+            // the candidate whose position in (value, slot) order is the remaining rank
+            for (int i = tid; i < c; i += kThreads) {
+                const int64_t v = S.cand_v[i];
+                int64_t pos = 0;
+                for (int j = 0; j < c; ++j) {
+                    const int64_t w = S.cand_v[j];
+                    pos += w < v || (w == v && j < i);
+                }
+                if (pos == r_in) P.p99[row] = v;
+            }
+            if (tid == 0) P.met[row] = met;
+            __syncthreads();
+            return;
+        }
     }
+    // ---- fallback: exact radix select over (TTFT - min) read from global memory
+    int64_t mn = INT64_MAX, mx = INT64_MIN;
+    for (int64_t k = tid; k < n; k += kThreads) {
+        const int64_t t = P.t_first[ob + k] - P.trace.arrival_us[tb + k];
+        mn = t < mn ? t : mn;
+        mx = t > mx ? t : mx;
+    }
+    mn = block_reduce<int64_t>(mn, INT64_MAX, [](int64_t a, int64_t b) { return a < b ? a : b; }, S.red64);
+    mx = block_reduce<int64_t>(mx, INT64_MIN, [](int64_t a, int64_t b) { return a > b ? a : b; }, S.red64);
+    const uint64_t range = (uint64_t)mx - (uint64_t)mn;
+    int shift = range == 0 ? 0 : 64 - __clzll((long long)range);  // bits still undetermined
+    uint64_t prefix = 0;                                            // chosen high bits of (ttft - mn)
+    int64_t rk = rank;                                              // rank among the candidates
+    while (shift > 0) {
+        const int dbits = shift < kDigit ? shift : kDigit;
+        const int above = shift;  // candidates agree with prefix on bits >= above
+        shift -= dbits;
+        for (int i = tid; i < kBins; i += kThreads) hist[i] = 0;
+        __syncthreads();
+        const uint32_t dmask = (1u << dbits) - 1u;
+        for (int64_t k = tid; k < n; k += kThreads) {
+            const uint64_t v = (uint64_t)(P.t_first[ob + k] - P.trace.arrival_us[tb + k]) - (uint64_t)mn;
+            const bool match = above >= 64 || (v >> above) == (prefix >> above);
+            if (match) atomicAdd(&hist[(uint32_t)(v >> shift) & dmask], 1u);
+        }
+        __syncthreads();
+        find_rank_bin(hist, kBins, rk, S.pick, S.wsum);
+        prefix |= (uint64_t)S.pick[0] << shift;
+        rk -= S.pick[1];
+        __syncthreads();
+    }
+    if (tid == 0) {
+        P.met[row] = met;
+        P.p99[row] = (int64_t)((uint64_t)mn + prefix);
+    }
+    __syncthreads();
+}
+
+template <int kRows, bool kStage, bool kHash>
+__global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParams P)
+{
+    __shared__ uint32_t hist[kRows][kLogBins];
+    __shared__ SelScratch S;
+    extern __shared__ uint16_t bin_s[];  // kStage: each row's TTFT bins, [kRows][n]
+    const int tid = threadIdx.x;
+    const int64_t n = P.n_req;
+    const int64_t rpr = P.rows_per_replica;
+    const int64_t upr = (rpr + kRows - 1) / kRows;  // units per replica
+    const int64_t n_units = (P.n_rows / rpr) * upr;
+
+    for (int64_t unit = blockIdx.x; unit < n_units; unit += gridDim.x) {
+        const int64_t rep = unit / upr;
+        const int64_t j0 = (unit - rep * upr) * kRows;
+        const int nr = (int)(rpr - j0 < kRows ? rpr - j0 : kRows);  // rows of this unit
+        const int64_t row0 = rep * rpr + j0;
+        const int64_t tb = rep * n;
+        if (kStage) {
+            for (int i = tid; i < kRows * kLogBins; i += kThreads) (&hist[0][0])[i] = 0;
+            __syncthreads();
+        }
+        int32_t met[kRows];
+        uint64_t h[kRows];  // kHash: each row's first-token and completion checksum terms
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) {
+            met[r] = 0;
+            h[r] = 0;
+        }
+        uint32_t wide = 0;  // bit r: row r has a TTFT outside [0, 2^32)
+        for (int64_t k = tid; k < n; k += kThreads) {
+            // every load of the request issued before any is used
+            const int64_t ta = __ldg(&P.trace.arrival_us[tb + k]);
+            const int64_t o = __ldg(&P.trace.true_out[tb + k]);
+            int c = (int)__ldg(&P.trace.slo_class[tb + k]);
+            int64_t tf[kRows], td[kRows];
+#pragma unroll
+            for (int r = 0; r < kRows; ++r) {
+                if (r < nr) {
+                    tf[r] = __ldg(&P.t_first[(row0 + r) * n + k]);
+                    td[r] = __ldg(&P.t_done[(row0 + r) * n + k]);
+                }
+            }
+            if (c >= P.n_classes) c = P.n_classes - 1;
+            const int64_t ttft_slo = P.ttft[c], tpot_slo = P.tpot[c] * (o - 1);
+            uint64_t m2 = 0, m3 = 0;  // the request-only halves of the checksum terms
+            if (kHash) {
+                m2 = mix64((uint64_t(2) << 56) ^ (uint64_t)k);
+                m3 = mix64((uint64_t(3) << 56) ^ (uint64_t)k);
+            }
+#pragma unroll
+            for (int r = 0; r < kRows; ++r) {
+                if (r < nr) {
+                    const int64_t ttft = tf[r] - ta;
+                    met[r] += ttft <= ttft_slo && (o == 1 || td[r] - tf[r] <= tpot_slo);
+                    const bool fits = (uint64_t)ttft < (uint64_t(1) << 32);
+                    wide |= (uint32_t)!fits << r;
+                    if (kStage) {
+                        const uint32_t b = fits ? log_bin((uint32_t)ttft) : 0u;
+                        atomicAdd(&hist[r][b], 1u);
+                        bin_s[(int64_t)r * n + k] = (uint16_t)b;
+                    }
+                    if (kHash) h[r] += mix64(m2 ^ (uint64_t)tf[r]) + mix64(m3 ^ (uint64_t)td[r]);
+                }
+            }
+        }
+        wide = (uint32_t)block_reduce<int32_t>((int32_t)wide, 0, [](int32_t a, int32_t b) { return a | b; },
+                                               reinterpret_cast<int32_t*>(S.red64));
+#pragma unroll
+        for (int r = 0; r < kRows; ++r) {
+            if (r < nr) {
+                const int32_t m_r = block_reduce<int32_t>(met[r], 0, [](int32_t a, int32_t b) { return a + b; },
+                                                          reinterpret_cast<int32_t*>(S.red64));
+                const int64_t row = row0 + r;
+                if (kHash) {
+                    const uint64_t h_r = (uint64_t)block_reduce<int64_t>((int64_t)h[r], 0, [](int64_t a, int64_t b) {
+                        return (int64_t)((uint64_t)a + (uint64_t)b);  // sum mod 2^64
+                    }, S.red64);
+                    if (tid == 0 && P.row_status[row] == CTR_OK) P.row_hash[row] += h_r;  // a failed row keeps 0
+                }
+                if (n == 0) {
+                    if (tid == 0) {
+                        P.met[row] = 0;
+                        P.p99[row] = -1;
+                    }
+                    continue;
+                }
+                select_row(P, row, tb, n, m_r, kStage && !((wide >> r) & 1u), hist[r], bin_s + (int64_t)r * n, S);
+            }
+        }
+    }
+}
+
+template <int kRows, bool kStage>
+cudaError_t launch_rows(const GoodputParams& p, int64_t dyn_bytes, bool hash, int sms, cudaStream_t stream)
+{
+    const void* k = hash ? (const void*)goodput_kernel<kRows, kStage, true>
+                         : (const void*)goodput_kernel<kRows, kStage, false>;
+    cudaError_t err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn_bytes);
+    if (err != cudaSuccess) return err;
+    int per_sm = 0;
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kThreads, (size_t)dyn_bytes);
+    if (err != cudaSuccess) return err;
+    const int64_t rpr = p.rows_per_replica;
+    int64_t blocks = (p.n_rows / rpr) * ((rpr + kRows - 1) / kRows);
+    const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+    if (blocks > cap) blocks = cap;
+    if (hash)
+        goodput_kernel<kRows, kStage, true><<<(unsigned)blocks, kThreads, (size_t)dyn_bytes, stream>>>(p);
+    else
+        goodput_kernel<kRows, kStage, false><<<(unsigned)blocks, kThreads, (size_t)dyn_bytes, stream>>>(p);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -251,32 +311,18 @@ cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream)
     if (err != cudaSuccess) return err;
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
-    constexpr int64_t kStageMaxBytes = 200 * 1024;  // a row's TTFT bins staged in shared memory up to this
-    const int64_t stage_bytes = p.n_req * 2;
+    // Two blocks per SM when a unit's staged bins, histograms and scratch fit in half the shared memory;
+    // two rows per unit when the replica has them (their request-only checksum mixes are shared).
+    constexpr int64_t kSmemBudget = 108 * 1024;
+    const int64_t fixed = (int64_t)sizeof(SelScratch) + 256;
     const bool hash = p.row_hash != nullptr;
-    if (stage_bytes > 0 && stage_bytes <= kStageMaxBytes) {
-        const void* k = hash ? (const void*)goodput_kernel<true, true> : (const void*)goodput_kernel<true, false>;
-        err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)stage_bytes);
-        if (err != cudaSuccess) return err;
-        int per_sm = 0;
-        err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kThreads, (size_t)stage_bytes);
-        if (err != cudaSuccess) return err;
-        int64_t blocks = p.n_rows;
-        const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
-        if (blocks > cap) blocks = cap;
-        if (hash)
-            goodput_kernel<true, true><<<(unsigned)blocks, kThreads, (size_t)stage_bytes, stream>>>(p);
-        else
-            goodput_kernel<true, false><<<(unsigned)blocks, kThreads, (size_t)stage_bytes, stream>>>(p);
-        return cudaGetLastError();
-    }
-    int64_t blocks = p.n_rows;
-    if (blocks > (int64_t)sms * 8) blocks = (int64_t)sms * 8;
-    if (hash)
-        goodput_kernel<false, true><<<(unsigned)blocks, kThreads, 0, stream>>>(p);
-    else
-        goodput_kernel<false, false><<<(unsigned)blocks, kThreads, 0, stream>>>(p);
-    return cudaGetLastError();
+    const int64_t n2 = p.n_req * 2;
+    auto fits = [&](int rows) { return n2 > 0 && rows * (n2 + 4 * kLogBins) + fixed <= kSmemBudget; };
+    if (p.rows_per_replica >= 2 && fits(2)) return launch_rows<2, true>(p, 2 * n2, hash, sms, stream);
+    if (fits(1)) return launch_rows<1, true>(p, n2, hash, sms, stream);
+    constexpr int64_t kStageMaxBytes = 200 * 1024;  // one row staged, one block per SM
+    if (n2 > 0 && n2 + 4 * kLogBins + fixed <= kStageMaxBytes) return launch_rows<1, true>(p, n2, hash, sms, stream);
+    return launch_rows<1, false>(p, 0, hash, sms, stream);  // rows too long to stage
 }
 
 }  // namespace ctr

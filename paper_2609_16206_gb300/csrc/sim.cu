@@ -26,7 +26,7 @@
 // Per-lane structures live in the workspace slot of the warp, each lane's
 // entries contiguous (a heap's top levels then share cache lines; the heaps
 // are 4-ary, a node's four children two 16-byte words and a heap of n keys
-// about log4 n levels deep, except with batched prefill: see HeapShape): a min-heap of
+// about log4 n levels deep, except with batched prefill: see heap_push_bin): a min-heap of
 // pending KV-ready keys (t_ready << 23 | k) per decode lane (the prefill
 // lanes use the same region as their in-flight ring of prefill end times,
 // packed with the prompt length as end << 21 | p), a min-heap of active
@@ -112,81 +112,130 @@ __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
     return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
-// Entries per lane of a heap region holding up to cap keys, for either arity below:
-// cap + 3 entries rounded up to 4 (a 32-byte multiple).
+// Entries per lane of a heap region holding up to cap keys.  The heaps are
+// 4-ary: node j (0-based) sits at position j + 3, so its children 4j + 1 ..
+// 4j + 4 sit at positions 4j + 4 .. 4j + 7, a 32-byte aligned block read as
+// two 16-byte words; the region has cap + 3 entries rounded up to 4.
 __host__ __device__ __forceinline__ int64_t heap_stride(int64_t cap) { return (cap + 6) & ~int64_t(3); }
 
-// Min-heaps of unique 64-bit keys, each lane's heap contiguous.  kArity 4: node j
-// (0-based) at position j + 3, its children 4j + 1 .. 4j + 4 at positions
-// 4j + 4 .. 4j + 7, one 32-byte aligned block read as two 16-byte words, about
-// log4 n levels: fewer dependent loads per pop, more compares per level.  kArity
-// 2: 1-based, children 2i and 2i + 1 one 16-byte word.  The kernel takes 4 for
-// long decode batches (the replica sweep's and the large pool's: -2 % and -6 %
-// there) and 2 with batched prefill, whose short-output document workload keeps
-// the batches small (4-ary is 6 % slower there).
-template <int kArity>
-struct HeapShape {
-    static constexpr int kRoot = kArity == 4 ? 3 : 1;
-    __device__ static __forceinline__ int parent(int i) { return kArity == 4 ? (i >> 2) + 2 : i >> 1; }
-    __device__ static __forceinline__ int first_child(int i) { return kArity == 4 ? (i - 2) << 2 : i << 1; }
-};
+constexpr int kHeapRoot = 3;
 
-template <int kArity>
+// min-heap of unique 64-bit keys; each lane's heap is contiguous
 __device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
 {
-    using S = HeapShape<kArity>;
-    int i = S::kRoot + n++;
-    while (i > S::kRoot) {
-        const int parent = S::parent(i);
+    int i = kHeapRoot + n++;
+    while (i > kHeapRoot) {
+        const int parent = (i >> 2) + 2;
         const uint64_t pv = h[parent];
         if (pv < key) break;
         h[i] = pv;
         i = parent;
     }
     h[i] = key;
-    if (i == S::kRoot) top = key;
+    if (i == kHeapRoot) top = key;
 }
 
-template <int kArity>
 __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
 {
-    using S = HeapShape<kArity>;
     const int m = n--;  // the last key moves into the hole left at the root
     if (m == 1) {
         top = kEmpty;
         return;
     }
-    const int lastp = S::kRoot + m - 1;
+    const int lastp = kHeapRoot + m - 1;
     const uint64_t last = h[lastp];
     const int endp = lastp - 1;  // position of the last key that stays
-    int i = S::kRoot;
+    int i = kHeapRoot;
     for (;;) {
-        const int c = S::first_child(i);
+        const int c = (i - 2) << 2;  // first child
         if (c > endp) break;
         const ulonglong2 c01 = *reinterpret_cast<const ulonglong2*>(h + c);
+        const ulonglong2 c23 = *reinterpret_cast<const ulonglong2*>(h + c + 2);
         uint64_t cv = c01.x;
         int ci = c;
         if (c + 1 <= endp && c01.y < cv) {
             cv = c01.y;
             ci = c + 1;
         }
-        if (kArity == 4) {
-            const ulonglong2 c23 = *reinterpret_cast<const ulonglong2*>(h + c + 2);
-            if (c + 2 <= endp && c23.x < cv) {
-                cv = c23.x;
-                ci = c + 2;
-            }
-            if (c + 3 <= endp && c23.y < cv) {
-                cv = c23.y;
-                ci = c + 3;
-            }
+        if (c + 2 <= endp && c23.x < cv) {
+            cv = c23.x;
+            ci = c + 2;
+        }
+        if (c + 3 <= endp && c23.y < cv) {
+            cv = c23.y;
+            ci = c + 3;
         }
         if (last < cv) break;
         h[i] = cv;
         i = ci;
     }
     h[i] = last;
-    top = h[S::kRoot];
+    top = h[kHeapRoot];
+}
+
+// Binary 1-based variants (children 2i and 2i + 1 in one 16-byte word), kept
+// for batched prefill: its short-output document workload keeps decode batches
+// small, where the extra compares of a 4-ary level cost more than the saved
+// levels (4,096 x 10,000: 97.6 ms binary, 104.1 ms 4-ary; the replica sweep and
+// the large pool are 2 % and 6 % faster 4-ary).  Same region stride.
+__device__ __forceinline__ void heap_push_bin(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
+{
+    int i = ++n;
+    while (i > 1) {
+        const int parent = i >> 1;
+        const uint64_t pv = h[parent];
+        if (pv < key) break;
+        h[i] = pv;
+        i = parent;
+    }
+    h[i] = key;
+    if (i == 1) top = key;
+}
+
+__device__ __forceinline__ void heap_pop_bin(uint64_t* h, int32_t& n, uint64_t& top)
+{
+    const int m = n--;
+    if (m == 1) {
+        top = kEmpty;
+        return;
+    }
+    const uint64_t last = h[m];
+    const int sz = m - 1;
+    int i = 1;
+    for (;;) {
+        const int c = 2 * i;
+        if (c > sz) break;
+        const ulonglong2 ch = *reinterpret_cast<const ulonglong2*>(h + c);  // c even: a 16-byte word
+        uint64_t cv = ch.x;
+        int ci = c;
+        if (c < sz && ch.y < cv) {
+            cv = ch.y;
+            ci = c + 1;
+        }
+        if (last < cv) break;
+        h[i] = cv;
+        i = ci;
+    }
+    h[i] = last;
+    top = h[1];
+}
+
+// the heap operations of a kernel instantiation: binary with batched prefill, else 4-ary
+template <bool kBin>
+__device__ __forceinline__ void hpush(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
+{
+    if constexpr (kBin)
+        heap_push_bin(h, n, top, key);
+    else
+        heap_push(h, n, top, key);
+}
+template <bool kBin>
+__device__ __forceinline__ void hpop(uint64_t* h, int32_t& n, uint64_t& top)
+{
+    if constexpr (kBin)
+        heap_pop_bin(h, n, top);
+    else
+        heap_pop(h, n, top);
 }
 
 // argmin over the lanes of 64-bit values (ties -> lowest lane)
@@ -219,7 +268,7 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
 {
     while (s.pend_n > 0 && (int64_t)(s.pend_top >> kKeyBits) <= t) {
         const uint32_t k = (uint32_t)(s.pend_top & kKeyMask);
-        heap_pop<kArity>(pend, s.pend_n, s.pend_top);
+        hpop<kArity == 2>(pend, s.pend_n, s.pend_top);
         if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
         int pos = s.w_head + s.w_n;
         if (pos >= P.cap_wait) pos -= P.cap_wait;
@@ -311,7 +360,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.stepping = false;
             while (s.n_act > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
                 const int64_t k = (int64_t)(s.act_top & kKeyMask);
-                heap_pop<kArity>(act, s.n_act, s.act_top);
+                hpop<kArity == 2>(act, s.n_act, s.act_top);
                 const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
                 const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
                 s.q -= 1;
@@ -338,7 +387,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 s.w_n -= 1;
                 s.kv_rsv += (int32_t)(pk + ok);
                 s.kv_res += (int32_t)pk;
-                heap_push<kArity>(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
+                hpush<kArity == 2>(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
                 admitted += 1;
             }
             if (s.n_act > 0) {
@@ -426,7 +475,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
 {
     constexpr bool kSig = kMode >= 1;  // the proxy's signals: ledger backlog, polled occupancy
     constexpr bool kBat = kMode == 2;  // batched prefill
-    constexpr int kArity = kBat ? 2 : 4;  // heap arity (see HeapShape)
+    constexpr int kArity = kBat ? 2 : 4;  // heap arity: binary with batched prefill (see heap_push_bin)
     constexpr int kRowsPerWarp = 32 / G;
     const int lane = threadIdx.x & 31;
     const int grp = lane / G;
@@ -549,7 +598,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 if (s.pend_n == P.cap_pend_store) {
                                     err = CTR_EOVERFLOW;  // the waiting FIFO has overflowed
                                 } else {
-                                    heap_push<kArity>(pend, s.pend_n, s.pend_top,
+                                    hpush<kArity == 2>(pend, s.pend_n, s.pend_top,
                                               ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift));
                                 }
                             }
@@ -759,7 +808,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         (ready >= 0 && s.pend_n == P.cap_pend_store)) {
                         err = CTR_EOVERFLOW;
                     } else {
-                        if (ready >= 0) heap_push<kArity>(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
+                        if (ready >= 0) hpush<kArity == 2>(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
                         s.q += 1;
                         s.sum += sum_is_o_hat ? ohk : ok;
                     }
