@@ -306,8 +306,17 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     if (e != cudaSuccess) return CTR_ECUDA;
     const int blocks = (int)((slots + wpb - 1) / wpb);
     const bool goodput = met_count != nullptr;
-    e = launch_sim(p, blocks, wpb, !goodput, s);
-    if (e != cudaSuccess || !goodput) return cuda_status(e);
+    e = launch_sim(p, blocks, wpb, s);
+    if (e != cudaSuccess) return cuda_status(e);
+    // Once the simulation has ended its per-warp structures are dead, so the slots hold, when they have
+    // room, the table of the checksum terms' request-only halves for the pass that follows.
+    uint64_t* kmix = nullptr;
+    if (n_rows > 0 && n_req > 0 && slots * p.slot_bytes >= 16 * n_req) {
+        kmix = reinterpret_cast<uint64_t*>(p.ws);
+        e = launch_mix_table(kmix, n_req, s);
+        if (e != cudaSuccess) return cuda_status(e);
+    }
+    if (!goodput) return cuda_status(launch_hash(p, kmix, blocks, s));
     // each row's goodput, in the same pass that adds its checksum's first-token and completion terms
     GoodputParams g;
     std::memset(&g, 0, sizeof(g));
@@ -326,6 +335,7 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     g.p99 = p99_ttft_us;
     g.row_hash = row_hash;
     g.row_status = row_status;
+    g.kmix = kmix;
     return cuda_status(launch_goodput(g, s));
 }
 

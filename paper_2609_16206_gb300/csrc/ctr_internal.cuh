@@ -118,9 +118,15 @@ struct SimParams {
 int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr);
 int sim_max_resident_warps(int* warps_per_block, int* blocks);
 int sim_group_width(int n_instances);  // lanes per simulated row; 32 / width rows share a warp
-// hash_pass: add the first-token and completion checksum terms in a pass of
-// their own (false when the goodput pass that follows adds them)
-cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, bool hash_pass, cudaStream_t stream);
+cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream);
+// The first-token and completion checksum terms in a pass of their own (when no
+// goodput pass adds them); kmix as for GoodputParams, or null.
+cudaError_t launch_hash(const SimParams& p, const uint64_t* kmix, int blocks, cudaStream_t stream);
+// The request-only halves of the checksum's first-token and completion terms:
+// t[k] = mix64((2 << 56) ^ k) and t[n + k] = mix64((3 << 56) ^ k) for k < n,
+// shared by every row of a call (the passes that sum the terms read them
+// instead of mixing each row-request's index again).
+cudaError_t launch_mix_table(uint64_t* t, int64_t n, cudaStream_t stream);
 
 // ---------------------------------------------------------------- goodput
 struct GoodputParams {
@@ -136,6 +142,7 @@ struct GoodputParams {
     // checksum terms to row_hash in the same pass over the outputs
     uint64_t* row_hash;
     const int32_t* row_status;
+    const uint64_t* kmix;  // optional with row_hash: the table of launch_mix_table for n_req
 };
 cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream);
 

@@ -234,8 +234,13 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
             const int64_t ttft_slo = P.ttft[c], tpot_slo = P.tpot[c] * (o - 1);
             uint64_t m2 = 0, m3 = 0;  // the request-only halves of the checksum terms
             if (kHash) {
-                m2 = mix64((uint64_t(2) << 56) ^ (uint64_t)k);
-                m3 = mix64((uint64_t(3) << 56) ^ (uint64_t)k);
+                if (P.kmix) {  // mixed once per call (launch_mix_table)
+                    m2 = __ldg(&P.kmix[k]);
+                    m3 = __ldg(&P.kmix[n + k]);
+                } else {
+                    m2 = mix64((uint64_t(2) << 56) ^ (uint64_t)k);
+                    m3 = mix64((uint64_t(3) << 56) ^ (uint64_t)k);
+                }
             }
 #pragma unroll
             for (int r = 0; r < kRows; ++r) {
@@ -280,6 +285,15 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
     }
 }
 
+__global__ void __launch_bounds__(256) mix_table_kernel(uint64_t* t, int64_t n)
+{
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < 2 * n; i += (int64_t)gridDim.x * blockDim.x) {
+        const bool first = i < n;
+        const int64_t k = first ? i : i - n;
+        t[i] = mix64(((first ? uint64_t(2) : uint64_t(3)) << 56) ^ (uint64_t)k);
+    }
+}
+
 template <int kRows, bool kStage>
 cudaError_t launch_rows(const GoodputParams& p, int64_t dyn_bytes, bool hash, int sms, cudaStream_t stream)
 {
@@ -302,6 +316,15 @@ cudaError_t launch_rows(const GoodputParams& p, int64_t dyn_bytes, bool hash, in
 }
 
 }  // namespace
+
+cudaError_t launch_mix_table(uint64_t* t, int64_t n, cudaStream_t stream)
+{
+    if (n <= 0) return cudaSuccess;
+    int64_t blocks = (2 * n + 255) / 256;
+    if (blocks > 4096) blocks = 4096;
+    mix_table_kernel<<<(unsigned)blocks, 256, 0, stream>>>(t, n);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream)
 {

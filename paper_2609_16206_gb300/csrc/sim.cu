@@ -853,7 +853,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
 // row over the simulator's outputs (coalesced; cheaper than hashing inside
 // the diverged event handlers).  Rows that failed keep the checksum 0.
 constexpr int kHashThreads = 256;
-__global__ void __launch_bounds__(kHashThreads) hash_kernel(const __grid_constant__ SimParams P)
+__global__ void __launch_bounds__(kHashThreads) hash_kernel(const __grid_constant__ SimParams P, const uint64_t* kmix)
 {
     __shared__ uint64_t part[kHashThreads / 32];
     for (int64_t row = blockIdx.x; row < P.n_rows; row += gridDim.x) {
@@ -864,7 +864,10 @@ __global__ void __launch_bounds__(kHashThreads) hash_kernel(const __grid_constan
         for (int64_t k = threadIdx.x; k < P.n_req; k += kHashThreads) {
             const int64_t tf = __ldcs(&P.t_first[ob + k]);
             const int64_t td = __ldcs(&P.t_done[ob + k]);
-            h += hterm(k, 2, (uint64_t)tf) + hterm(k, 3, (uint64_t)td);
+            if (kmix)  // the request-only halves, mixed once per call (launch_mix_table)
+                h += mix64(__ldg(&kmix[k]) ^ (uint64_t)tf) + mix64(__ldg(&kmix[P.n_req + k]) ^ (uint64_t)td);
+            else
+                h += hterm(k, 2, (uint64_t)tf) + hterm(k, 3, (uint64_t)td);
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) h += __shfl_xor_sync(kFull, h, off);
@@ -956,7 +959,7 @@ cudaError_t launch_mode(const SimParams& p, int blocks, cudaStream_t stream)
 
 }  // namespace
 
-cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, bool hash_pass, cudaStream_t stream)
+cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, cudaStream_t stream)
 {
     (void)warps_per_block;
     bool signals = false;  // the proxy's ledger backlog or polled occupancy in some constant set
@@ -965,10 +968,14 @@ cudaError_t launch_sim(const SimParams& p, int blocks, int warps_per_block, bool
                           : signals       ? launch_mode<1>(p, blocks, stream)
                                           : launch_mode<0>(p, blocks, stream);
     if (e != cudaSuccess) return e;
-    if (hash_pass && p.n_rows > 0) {  // else the caller's goodput pass adds these terms
-        const int64_t hb = p.n_rows < (int64_t)blocks * 8 ? p.n_rows : (int64_t)blocks * 8;
-        hash_kernel<<<(unsigned)hb, kHashThreads, 0, stream>>>(p);
-    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_hash(const SimParams& p, const uint64_t* kmix, int blocks, cudaStream_t stream)
+{
+    if (p.n_rows == 0) return cudaSuccess;
+    const int64_t hb = p.n_rows < (int64_t)blocks * 8 ? p.n_rows : (int64_t)blocks * 8;
+    hash_kernel<<<(unsigned)hb, kHashThreads, 0, stream>>>(p, kmix);
     return cudaGetLastError();
 }
 
