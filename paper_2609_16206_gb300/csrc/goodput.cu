@@ -16,8 +16,9 @@
 // to stage falls back to a radix select over the exact TTFTs read from global
 // memory (11-bit digits, most significant first).  Called from ctr_simulate
 // with kHash, pass 0 also sums each row's checksum terms of first-token and
-// completion times; the request-only half of those terms is mixed once per
-// request for the unit's rows.
+// completion times; the request-only half of those terms is read from the
+// call's table (launch_mix_table) when ctr_simulate has one, else mixed once
+// per request for the unit's rows.
 #include "ctr_internal.cuh"
 
 namespace ctr {
@@ -335,7 +336,8 @@ cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream)
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
     // Two blocks per SM when a unit's staged bins, histograms and scratch fit in half the shared memory;
-    // two rows per unit when the replica has them (their request-only checksum mixes are shared).
+    // two rows per unit when the replica has them (they share the trace's reads and, without a table, the
+    // request-only checksum mixes).
     constexpr int64_t kSmemBudget = 108 * 1024;
     const int64_t fixed = (int64_t)sizeof(SelScratch) + 256;
     const bool hash = p.row_hash != nullptr;
