@@ -616,7 +616,7 @@ SIM_SLICE_COUNTERS: dict = {
 
 # DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.
 SCORE_DRAM_PER_LAUNCH: dict = {
-    "86ed7794a9408ef3": {"read": 9485312.0, "write": 0.0},
+    "59758572497f3adc": {"read": 9484800.0, "write": 0.0},
 }
 
 
