@@ -606,12 +606,12 @@ def run_ours(args, rank, world, local_rank):
 # per routed request, keyed by a hash of the simulator's code: a stale entry
 # (the kernel changed since the counters were taken) reports null.
 SIM_SLICE_COUNTERS: dict = {
-    "4a32a48f56cc50de": {"warp_inst_per_routed": 34162497367 / 81_920_000,
-                         "thread_inst_per_warp_inst": 281165272017 / 34162497367,
-                         "dram_bytes_per_routed": (2378798336 + 1562979840) / 81_920_000,
+    "110645194cd49beb": {"warp_inst_per_routed": 34162633267 / 81_920_000,
+                         "thread_inst_per_warp_inst": 281165931678 / 34162633267,
+                         "dram_bytes_per_routed": (2383195136 + 1564433152) / 81_920_000,
                          "slice": "ncu on one launch of 1,024 replicas x 20,000 requests x 4 policies "
                                   "(81.92 M routed requests): 3.416e10 warp-instructions, 2.812e11 thread-"
-                                  "instructions, 2.379 GB DRAM read + 1.563 GB written"},
+                                  "instructions, 2.383 GB DRAM read + 1.564 GB written"},
 }
 
 # DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.

@@ -30,6 +30,7 @@ extern "C" {
 #define CTR_ECUDA (-2)     /* CUDA launch / driver error */
 #define CTR_EOVERFLOW (-3) /* a fixed-capacity structure filled up, or a time reached 2^40 us */
 #define CTR_ETIMEOUT (-4)  /* the per-instance decode-step budget ran out */
+#define CTR_EBOUNDS (-5)   /* bounds-checked build only: an index fell outside its buffer (a library defect) */
 
 #define CTR_MAX_INSTANCES 32      /* prefill + decode instances of one simulated cluster */
 #define CTR_MAX_CLASSES 4         /* SLO classes */
@@ -277,6 +278,16 @@ const char* ctr_strerror(int code);
 /* ctr_abi_version -- increments on any change to the structs, the signatures or
  * the accepted ranges. */
 int ctr_abi_version(void);
+
+/* ctr_bounds_checked -- 1 in libctr_checked.so, 0 in libctr.so.  Both export
+ * the same entry points with the same results.  The checked build compiles the
+ * simulator's kernels (sim_kernel and its checksum pass) with a bounds check on
+ * every index into the workspace, the trace and the outputs: an index outside
+ * its buffer skips the access (a load reads 0) and the row ends with
+ * CTR_EBOUNDS in row_status (no fault, no trap).  With valid arguments that
+ * status never occurs; the checked build exists to show it on the GPU, where
+ * no memory checker runs.  It is slower and not meant for production. */
+int ctr_bounds_checked(void);
 
 #ifdef __cplusplus
 }

@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 6;
+constexpr int kAbiVersion = 7;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -73,6 +73,8 @@ extern "C" {
 
 int ctr_abi_version(void) { return kAbiVersion; }
 
+int ctr_bounds_checked(void) { return CTR_BOUNDS_CHECK; }
+
 const char* ctr_strerror(int code)
 {
     switch (code) {
@@ -81,6 +83,7 @@ const char* ctr_strerror(int code)
     case CTR_ECUDA: return "CUDA launch or driver error";
     case CTR_EOVERFLOW: return "a fixed-capacity structure filled up or a time reached 2^40 us";
     case CTR_ETIMEOUT: return "decode-step budget exhausted";
+    case CTR_EBOUNDS: return "an index fell outside its buffer (bounds-checked build)";
     default: return "unknown ctr status";
     }
 }
@@ -271,6 +274,8 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
     p.t_done = t_done_us;
     p.row_hash = row_hash;
     p.row_status = row_status;
+    p.trace_len = (int64_t)n_replicas * n_req;
+    p.out_len = n_rows * n_req;
     for (int i = 0; i < n_const_sets; ++i) {
         const ctr_cost_consts& k = consts[i];
         ConstsDev& d = p.sets[i];

@@ -9,6 +9,11 @@
 
 namespace ctr {
 
+// Bounds-checked builds (libctr_checked.so) define CTR_BOUNDS_CHECK=1.
+#ifndef CTR_BOUNDS_CHECK
+#define CTR_BOUNDS_CHECK 0
+#endif
+
 constexpr int kWarp = 32;
 constexpr int64_t kTimeLimit = int64_t(1) << 40;   // every simulated time stays below this
 constexpr int64_t kArrivalLimit = int64_t(1) << 39;
@@ -114,6 +119,8 @@ struct SimParams {
     uint64_t* row_hash;
     int32_t* row_status;
     ConstsDev sets[CTR_MAX_CONST_SETS];
+    int64_t trace_len;          // entries of each trace array (replicas x requests)
+    int64_t out_len;            // entries of each per-request output (rows x requests)
 };
 int64_t sim_slot_bytes(const ctr_sim_cfg& cfg, int64_t* off_act, int64_t* off_wait, int32_t* cap_pr);
 int sim_max_resident_warps(int* warps_per_block, int* blocks);

@@ -112,6 +112,48 @@ __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
     return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
+// Checked accesses.  A build with CTR_BOUNDS_CHECK=1 compares every index with
+// the length of its buffer first; an index outside skips the access (a load
+// gives 0) and sets `bad`, and the row ends with CTR_EBOUNDS.  Other builds
+// compile the plain access (the length and the flag are dead code there).
+#if CTR_BOUNDS_CHECK
+__device__ __forceinline__ bool ck_out(int64_t i, int64_t len, bool& bad)
+{
+    const bool out = (uint64_t)i >= (uint64_t)len;
+    bad = bad || out;
+    return out;
+}
+#define CTR_CK_OUT(i, len, bad) ck_out((int64_t)(i), (len), (bad))
+#else
+#define CTR_CK_OUT(i, len, bad) false
+#endif
+// (the index keeps the caller's type, so the unchecked address arithmetic is the plain one)
+template <typename T, typename I>
+__device__ __forceinline__ T ck_ld(const T* p, I i, int64_t len, bool& bad)
+{
+    if (CTR_CK_OUT(i, len, bad)) return T();
+    return p[i];
+}
+template <typename T, typename I>
+__device__ __forceinline__ T ck_ldg(const T* p, I i, int64_t len, bool& bad)  // read-only data
+{
+    if (CTR_CK_OUT(i, len, bad)) return T();
+    return __ldg(p + i);
+}
+template <typename T, typename I>
+__device__ __forceinline__ void ck_st(T* p, I i, int64_t len, T v, bool& bad)
+{
+    if (CTR_CK_OUT(i, len, bad)) return;
+    p[i] = v;
+}
+// entries i and i + 1 (i even) as one 16-byte word
+template <typename I>
+__device__ __forceinline__ ulonglong2 ck_ld2(const uint64_t* p, I i, int64_t len, bool& bad)
+{
+    if (CTR_CK_OUT(i, len - 1, bad)) return make_ulonglong2(0, 0);
+    return *reinterpret_cast<const ulonglong2*>(p + i);
+}
+
 // Entries per lane of a heap region holding up to cap keys.  The heaps are
 // 4-ary: node j (0-based) sits at position j + 3, so its children 4j + 1 ..
 // 4j + 4 sit at positions 4j + 4 .. 4j + 7, a 32-byte aligned block read as
@@ -121,21 +163,22 @@ __host__ __device__ __forceinline__ int64_t heap_stride(int64_t cap) { return (c
 constexpr int kHeapRoot = 3;
 
 // min-heap of unique 64-bit keys; each lane's heap is contiguous
-__device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
+__device__ __forceinline__ void heap_push(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key, int64_t lim,
+                                          bool& bad)
 {
     int i = kHeapRoot + n++;
     while (i > kHeapRoot) {
         const int parent = (i >> 2) + 2;
-        const uint64_t pv = h[parent];
+        const uint64_t pv = ck_ld(h, parent, lim, bad);
         if (pv < key) break;
-        h[i] = pv;
+        ck_st(h, i, lim, pv, bad);
         i = parent;
     }
-    h[i] = key;
+    ck_st(h, i, lim, key, bad);
     if (i == kHeapRoot) top = key;
 }
 
-__device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
+__device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top, int64_t lim, bool& bad)
 {
     const int m = n--;  // the last key moves into the hole left at the root
     if (m == 1) {
@@ -143,14 +186,14 @@ __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
         return;
     }
     const int lastp = kHeapRoot + m - 1;
-    const uint64_t last = h[lastp];
+    const uint64_t last = ck_ld(h, lastp, lim, bad);
     const int endp = lastp - 1;  // position of the last key that stays
     int i = kHeapRoot;
     for (;;) {
         const int c = (i - 2) << 2;  // first child
         if (c > endp) break;
-        const ulonglong2 c01 = *reinterpret_cast<const ulonglong2*>(h + c);
-        const ulonglong2 c23 = *reinterpret_cast<const ulonglong2*>(h + c + 2);
+        const ulonglong2 c01 = ck_ld2(h + c, 0, lim - c, bad);  // the block of four as two 16-byte words
+        const ulonglong2 c23 = ck_ld2(h + c, 2, lim - c, bad);
         uint64_t cv = c01.x;
         int ci = c;
         if (c + 1 <= endp && c01.y < cv) {
@@ -166,11 +209,11 @@ __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
             ci = c + 3;
         }
         if (last < cv) break;
-        h[i] = cv;
+        ck_st(h, i, lim, cv, bad);
         i = ci;
     }
-    h[i] = last;
-    top = h[kHeapRoot];
+    ck_st(h, i, lim, last, bad);
+    top = ck_ld(h, kHeapRoot, lim, bad);
 }
 
 // Binary 1-based variants (children 2i and 2i + 1 in one 16-byte word), kept
@@ -178,34 +221,35 @@ __device__ __forceinline__ void heap_pop(uint64_t* h, int32_t& n, uint64_t& top)
 // small, where the extra compares of a 4-ary level cost more than the saved
 // levels (4,096 x 10,000: 97.6 ms binary, 104.1 ms 4-ary; the replica sweep and
 // the large pool are 2 % and 6 % faster 4-ary).  Same region stride.
-__device__ __forceinline__ void heap_push_bin(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
+__device__ __forceinline__ void heap_push_bin(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key, int64_t lim,
+                                              bool& bad)
 {
     int i = ++n;
     while (i > 1) {
         const int parent = i >> 1;
-        const uint64_t pv = h[parent];
+        const uint64_t pv = ck_ld(h, parent, lim, bad);
         if (pv < key) break;
-        h[i] = pv;
+        ck_st(h, i, lim, pv, bad);
         i = parent;
     }
-    h[i] = key;
+    ck_st(h, i, lim, key, bad);
     if (i == 1) top = key;
 }
 
-__device__ __forceinline__ void heap_pop_bin(uint64_t* h, int32_t& n, uint64_t& top)
+__device__ __forceinline__ void heap_pop_bin(uint64_t* h, int32_t& n, uint64_t& top, int64_t lim, bool& bad)
 {
     const int m = n--;
     if (m == 1) {
         top = kEmpty;
         return;
     }
-    const uint64_t last = h[m];
+    const uint64_t last = ck_ld(h, m, lim, bad);
     const int sz = m - 1;
     int i = 1;
     for (;;) {
         const int c = 2 * i;
         if (c > sz) break;
-        const ulonglong2 ch = *reinterpret_cast<const ulonglong2*>(h + c);  // c even: a 16-byte word
+        const ulonglong2 ch = ck_ld2(h, c, lim, bad);  // c even: a 16-byte word
         uint64_t cv = ch.x;
         int ci = c;
         if (c < sz && ch.y < cv) {
@@ -213,29 +257,29 @@ __device__ __forceinline__ void heap_pop_bin(uint64_t* h, int32_t& n, uint64_t& 
             ci = c + 1;
         }
         if (last < cv) break;
-        h[i] = cv;
+        ck_st(h, i, lim, cv, bad);
         i = ci;
     }
-    h[i] = last;
-    top = h[1];
+    ck_st(h, i, lim, last, bad);
+    top = ck_ld(h, 1, lim, bad);
 }
 
 // the heap operations of a kernel instantiation: binary with batched prefill, else 4-ary
 template <bool kBin>
-__device__ __forceinline__ void hpush(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key)
+__device__ __forceinline__ void hpush(uint64_t* h, int32_t& n, uint64_t& top, uint64_t key, int64_t lim, bool& bad)
 {
     if constexpr (kBin)
-        heap_push_bin(h, n, top, key);
+        heap_push_bin(h, n, top, key, lim, bad);
     else
-        heap_push(h, n, top, key);
+        heap_push(h, n, top, key, lim, bad);
 }
 template <bool kBin>
-__device__ __forceinline__ void hpop(uint64_t* h, int32_t& n, uint64_t& top)
+__device__ __forceinline__ void hpop(uint64_t* h, int32_t& n, uint64_t& top, int64_t lim, bool& bad)
 {
     if constexpr (kBin)
-        heap_pop_bin(h, n, top);
+        heap_pop_bin(h, n, top, lim, bad);
     else
-        heap_pop(h, n, top);
+        heap_pop(h, n, top, lim, bad);
 }
 
 // argmin over the lanes of 64-bit values (ties -> lowest lane)
@@ -264,15 +308,16 @@ struct Decode {
 // Move every pending request whose KV is ready by t into the waiting FIFO, in
 // (time, index) order; the FIFO's size is checked after each insertion.
 template <int kArity>
-__device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams& P, uint64_t* pend, uint32_t* wait)
+__device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams& P, uint64_t* pend, uint32_t* wait,
+                                           bool& bad)
 {
     while (s.pend_n > 0 && (int64_t)(s.pend_top >> kKeyBits) <= t) {
         const uint32_t k = (uint32_t)(s.pend_top & kKeyMask);
-        hpop<kArity == 2>(pend, s.pend_n, s.pend_top);
+        hpop<kArity == 2>(pend, s.pend_n, s.pend_top, heap_stride(P.cap_pr), bad);
         if (s.w_n == P.cap_wait) return CTR_EOVERFLOW;
         int pos = s.w_head + s.w_n;
         if (pos >= P.cap_wait) pos -= P.cap_wait;
-        wait[pos] = k;
+        ck_st(wait, pos, P.cap_wait, k, bad);
         s.w_n += 1;
     }
     return CTR_OK;
@@ -287,7 +332,7 @@ __device__ __forceinline__ int flush_ready(Decode& s, int64_t t, const SimParams
 template <bool kSnap, int kArity>
 __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimParams& P, uint64_t* pend, uint64_t* act,
                                               uint32_t* wait, int64_t tb, int64_t ob, int64_t& tsnap, int64_t& kv_snap,
-                                              bool sum_is_o_hat)
+                                              bool sum_is_o_hat, bool& bad)
 {
     for (;;) {
         // Plain step ends first: the step ends by T, no request finishes with
@@ -360,34 +405,35 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
             s.stepping = false;
             while (s.n_act > 0 && (int32_t)(s.act_top >> kKeyBits) == s.step_idx) {
                 const int64_t k = (int64_t)(s.act_top & kKeyMask);
-                hpop<kArity == 2>(act, s.n_act, s.act_top);
-                const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
-                const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
+                hpop<kArity == 2>(act, s.n_act, s.act_top, heap_stride(P.cap_act), bad);
+                const int64_t pk = ck_ldg(P.trace.prompt_len, tb + k, P.trace_len, bad);
+                const int64_t ok = ck_ldg(P.trace.true_out, tb + k, P.trace_len, bad);
                 s.q -= 1;
                 s.kv_res -= (int32_t)(pk + ok);
                 s.kv_rsv -= (int32_t)(pk + ok);
-                if (sum_is_o_hat) s.sum -= __ldg(&P.trace.pred_out[tb + k]);
-                P.t_done[ob + k] = tev;
+                if (sum_is_o_hat) s.sum -= ck_ldg(P.trace.pred_out, tb + k, P.trace_len, bad);
+                ck_st(P.t_done, ob + k, P.out_len, tev, bad);
             }
         }
         // (2) every request KV-ready by now joins the waiting FIFO in (time, index) order
-        const int rc = flush_ready<kArity>(s, tev, P, pend, wait);
+        const int rc = flush_ready<kArity>(s, tev, P, pend, wait, bad);
         if (rc != CTR_OK) return rc;
         // (3) not mid-step: strict FCFS admission while the reservation fits, then start a step
         if (!s.stepping) {
             const int pos0 = s.w_head;
             int admitted = 0;
             while (s.w_n > 0) {
-                const uint32_t k = wait[s.w_head];
-                const int64_t pk = __ldg(&P.trace.prompt_len[tb + k]);
-                const int64_t ok = __ldg(&P.trace.true_out[tb + k]);
+                const uint32_t k = ck_ld(wait, s.w_head, P.cap_wait, bad);
+                const int64_t pk = ck_ldg(P.trace.prompt_len, tb + k, P.trace_len, bad);
+                const int64_t ok = ck_ldg(P.trace.true_out, tb + k, P.trace_len, bad);
                 if ((uint32_t)s.kv_rsv + (uint32_t)(pk + ok) > (uint32_t)P.kv_cap) break;  // < 2^31 + 2^21
                 if (s.n_act == P.cap_act) return CTR_EOVERFLOW;
                 s.w_head = s.w_head + 1 == P.cap_wait ? 0 : s.w_head + 1;
                 s.w_n -= 1;
                 s.kv_rsv += (int32_t)(pk + ok);
                 s.kv_res += (int32_t)pk;
-                hpush<kArity == 2>(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k);
+                hpush<kArity == 2>(act, s.n_act, s.act_top, ((uint64_t)(s.step_idx + ok) << kKeyBits) | k,
+                                   heap_stride(P.cap_act), bad);
                 admitted += 1;
             }
             if (s.n_act > 0) {
@@ -397,8 +443,8 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
                 s.stepping = true;
                 int pos = pos0;
                 for (int i = 0; i < admitted; ++i) {  // first token at the end of this step
-                    const uint32_t k = wait[pos];
-                    P.t_first[ob + k] = s.step_end;
+                    const uint32_t k = ck_ld(wait, pos, P.cap_wait, bad);
+                    ck_st(P.t_first, ob + k, P.out_len, s.step_end, bad);
                     pos = pos + 1 == P.cap_wait ? 0 : pos + 1;
                 }
             }
@@ -408,7 +454,7 @@ __device__ __forceinline__ int decode_advance(Decode& s, int64_t T, const SimPar
 }
 
 // Per-request bounds, arrival order (CTR_EINVAL before anything is simulated).
-__device__ __forceinline__ bool row_valid(const SimParams& P, int64_t tb, int lane)
+__device__ __forceinline__ bool row_valid(const SimParams& P, int64_t tb, int lane, bool& bad)
 {
     int64_t prev_last = 0;
     for (int64_t base = 0; base < P.n_req; base += 32) {
@@ -417,11 +463,11 @@ __device__ __forceinline__ bool row_valid(const SimParams& P, int64_t tb, int la
         int64_t t = 0;
         bool bad = false;
         if (live) {
-            t = P.trace.arrival_us[tb + k];
-            const int64_t p = P.trace.prompt_len[tb + k];
-            const int64_t o = P.trace.true_out[tb + k];
-            const int64_t oh = P.trace.pred_out[tb + k];
-            const int64_t c = P.trace.slo_class[tb + k];
+            t = ck_ld(P.trace.arrival_us, tb + k, P.trace_len, bad);
+            const int64_t p = ck_ld(P.trace.prompt_len, tb + k, P.trace_len, bad);
+            const int64_t o = ck_ld(P.trace.true_out, tb + k, P.trace_len, bad);
+            const int64_t oh = ck_ld(P.trace.pred_out, tb + k, P.trace_len, bad);
+            const int64_t c = ck_ld(P.trace.slo_class, tb + k, P.trace_len, bad);
             bad = t < 0 || t >= kArrivalLimit || p < 0 || p > (1 << 20) || o < 1 || o > (1 << 20) ||
                   p + o > P.kv_cap || oh < 0 || oh > (1 << 17) || c >= P.n_classes;
         }
@@ -514,11 +560,14 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         const int64_t ob = row * n;
 
         // per-request bounds, one row at a time with the whole warp
+        bool oob = false;  // bounds-checked builds: an index of this lane fell outside its buffer
         bool valid = false;
         for (int g = 0; g < kRowsPerWarp; ++g) {
             const int64_t r = base_row + g;
             if (r >= P.n_rows) break;
-            const bool ok = row_valid(P, (r / per_rep) * n, lane);
+            bool oob_g = false;
+            const bool ok = row_valid(P, (r / per_rep) * n, lane, oob_g);
+            if (g == grp) oob = oob_g;
             if (g == grp) valid = ok;
         }
         bool live = has_row && valid;
@@ -563,7 +612,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         int pos = ring_head;
                         int64_t pmax = 0;
                         while (run_n < ring_n) {
-                            const int64_t pj = ring[pos] & kRingPMask;
+                            const int64_t pj = ck_ld(ring, pos, (int64_t)P.cap_ring, oob) & kRingPMask;
                             if (run_n > 0 && run_p + pj > P.pre_batch) break;
                             run_p += pj;
                             pmax = pj > pmax ? pj : pmax;
@@ -592,14 +641,15 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     if (is_dec && live) {
                         int pos = h_i;
                         for (int32_t m = 0; m < m_i; ++m) {
-                            const int64_t v = rings[src * pr_stride + pos];
+                            const int64_t v = ck_ld(rings + src * pr_stride, pos, (int64_t)P.cap_ring, oob);
                             if ((int)((v >> kRingPBits) & 31) == gl - P.n_pre) {
                                 const int64_t ready = e_i + P.xfer_tok * (v & kRingPMask);
                                 if (s.pend_n == P.cap_pend_store) {
                                     err = CTR_EOVERFLOW;  // the waiting FIFO has overflowed
                                 } else {
                                     hpush<kArity == 2>(pend, s.pend_n, s.pend_top,
-                                              ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift));
+                                              ((uint64_t)ready << kKeyBits) | (uint64_t)(v >> kRingKShift), pr_stride,
+                                              oob);
                                 }
                             }
                             pos = pos + 1 == P.cap_ring ? 0 : pos + 1;
@@ -616,10 +666,11 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
             int64_t my_t = 0;
             uint32_t my_pc = 0, my_o = 0, my_oh = 0;
             if (mine) {
-                my_t = P.trace.arrival_us[tb + kl];
-                my_pc = (uint32_t)P.trace.prompt_len[tb + kl] | ((uint32_t)P.trace.slo_class[tb + kl] << 24);
-                my_o = (uint32_t)P.trace.true_out[tb + kl];
-                my_oh = (uint32_t)P.trace.pred_out[tb + kl];
+                my_t = ck_ld(P.trace.arrival_us, tb + kl, P.trace_len, oob);
+                my_pc = (uint32_t)ck_ld(P.trace.prompt_len, tb + kl, P.trace_len, oob) |
+                        ((uint32_t)ck_ld(P.trace.slo_class, tb + kl, P.trace_len, oob) << 24);
+                my_o = (uint32_t)ck_ld(P.trace.true_out, tb + kl, P.trace_len, oob);
+                my_oh = (uint32_t)ck_ld(P.trace.pred_out, tb + kl, P.trace_len, oob);
             }
             uint32_t my_route = 0;
             const int cnt = (int)(n - base < G ? n - base : G);
@@ -643,14 +694,17 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                                 last_poll = tp;
                             }
                         }
-                        if (err == CTR_OK) err = decode_advance<kSig, kArity>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen, sum_is_o_hat);
+                        if (err == CTR_OK)
+                            err = decode_advance<kSig, kArity>(s, T, P, pend, act, wait, tb, ob, tsnap, kv_seen,
+                                                               sum_is_o_hat, oob);
                     } else if (is_pre && !batched) {
                         const int64_t thr = ((T + 1) << kRingPBits) - 1;  // entries whose prefill ended by T
                         while (ring_n > 0 && ring_front <= (uint64_t)thr) {
                             if constexpr (kSig) ring_sum_p -= ring_front & kRingPMask;
                             ring_head = ring_head + 1 == P.cap_ring ? 0 : ring_head + 1;
                             ring_n -= 1;
-                            ring_front = ring_n > 0 ? (uint64_t)ring[ring_head] : (uint64_t)kNever;
+                            ring_front = ring_n > 0 ? (uint64_t)ck_ld(ring, ring_head, (int64_t)P.cap_ring, oob)
+                                                    : (uint64_t)kNever;
                         }
                         if (ring_n == 0) ring_head = 0;
                     }
@@ -761,7 +815,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                     } else {
                         int pos = ring_head + ring_n;
                         if (pos >= P.cap_ring) pos -= P.cap_ring;
-                        ring[pos] = (k << kRingKShift) | ((int64_t)id << kRingPBits) | pk;
+                        ck_st(ring, pos, (int64_t)P.cap_ring, (k << kRingKShift) | ((int64_t)id << kRingPBits) | pk, oob);
                         ring_n += 1;
                         ring_sum_p += pk;
                         if (run_n == 0) {  // an idle instance starts a batch of this request at once
@@ -793,7 +847,7 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                         int pos = ring_head + ring_n;
                         if (pos >= P.cap_ring) pos -= P.cap_ring;
                         const int64_t e = (end << kRingPBits) | pk;
-                        ring[pos] = e;
+                        ck_st(ring, pos, (int64_t)P.cap_ring, e, oob);
                         if (ring_n == 0) ring_front = (uint64_t)e;
                         ring_n += 1;
                         if constexpr (kSig) ring_sum_p += pk;
@@ -803,12 +857,14 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 if (live && gl == P.n_pre + id && ready < kTimeLimit) {
                     // requests routed here whose KV is not ready yet, exactly: first move
                     // those already ready (kept in the heap until the step end) if it matters
-                    if (s.q - s.w_n - s.n_act >= P.cap_pend) err = flush_ready<kArity>(s, T, P, pend, wait);
+                    if (s.q - s.w_n - s.n_act >= P.cap_pend) err = flush_ready<kArity>(s, T, P, pend, wait, oob);
                     if (err != CTR_OK || s.q - s.w_n - s.n_act == P.cap_pend ||
                         (ready >= 0 && s.pend_n == P.cap_pend_store)) {
                         err = CTR_EOVERFLOW;
                     } else {
-                        if (ready >= 0) hpush<kArity == 2>(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k);
+                        if (ready >= 0)
+                            hpush<kArity == 2>(pend, s.pend_n, s.pend_top, ((uint64_t)ready << kKeyBits) | (uint64_t)k,
+                                               pr_stride, oob);
                         s.q += 1;
                         s.sum += sum_is_o_hat ? ohk : ok;
                     }
@@ -820,8 +876,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
                 // the routing term of the row checksum, all lanes at once (the
                 // first-token and completion terms are added by hash_kernel)
                 h += hterm(kl, 1, (uint64_t)my_route);
-                if (P.i_pre) P.i_pre[ob + kl] = (uint8_t)(my_route >> 8);
-                if (P.i_dec) P.i_dec[ob + kl] = (uint8_t)(my_route & 0xFF);
+                if (P.i_pre) ck_st(P.i_pre, ob + kl, P.out_len, (uint8_t)(my_route >> 8), oob);
+                if (P.i_dec) ck_st(P.i_dec, ob + kl, P.out_len, (uint8_t)(my_route & 0xFF), oob);
             }
         }
         // drain: every remaining batch, then every remaining event
@@ -833,7 +889,8 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         }
         if (live && is_dec) {
             int64_t no_snap = -1;
-            err = decode_advance<false, kArity>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, sum_is_o_hat);
+            err = decode_advance<false, kArity>(s, kNever - 1, P, pend, act, wait, tb, ob, no_snap, kv_seen, sum_is_o_hat,
+                                                oob);
         }
 
 #pragma unroll
@@ -842,6 +899,9 @@ __global__ void __launch_bounds__(kWarpsPerBlock * 32, kBlocksPerSM) sim_kernel(
         if (__ballot_sync(kFull, err == CTR_ETIMEOUT) & gmask) status = CTR_ETIMEOUT;
         if (__ballot_sync(kFull, err == CTR_EOVERFLOW) & gmask) status = CTR_EOVERFLOW;
         if (has_row && !valid) status = CTR_EINVAL;
+#if CTR_BOUNDS_CHECK
+        if (__ballot_sync(kFull, oob) & gmask) status = CTR_EBOUNDS;
+#endif
         if (gl == 0 && has_row) {
             P.row_status[row] = status;
             P.row_hash[row] = status == CTR_OK ? h : 0;

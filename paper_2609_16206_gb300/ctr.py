@@ -16,8 +16,10 @@ import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libctr.so")
+# the bounds-checked build of the same library (build.build(checked=True)); use_library() switches to it
+LIB_CHECKED_PATH = os.path.join(_HERE, "libctr_checked.so")
 
-CTR_OK, CTR_EINVAL, CTR_ECUDA, CTR_EOVERFLOW, CTR_ETIMEOUT = 0, -1, -2, -3, -4
+CTR_OK, CTR_EINVAL, CTR_ECUDA, CTR_EOVERFLOW, CTR_ETIMEOUT, CTR_EBOUNDS = 0, -1, -2, -3, -4, -5
 CTR_MAX_INSTANCES = 32
 CTR_MAX_CONST_SETS = 128
 CTR_MAX_REQUESTS = 1 << 23
@@ -105,8 +107,21 @@ def lib():
             L.ctr_strerror.argtypes = [C.c_int]
             L.ctr_strerror.restype = C.c_char_p
             L.ctr_abi_version.restype = C.c_int
+            L.ctr_bounds_checked.restype = C.c_int
             _lib = L
     return _lib
+
+
+def use_library(path: str) -> str:
+    """Make every following call go to the library at `path` (LIB_PATH or
+    LIB_CHECKED_PATH); returns the path in use before."""
+    global _lib, LIB_PATH
+    with _lock:
+        before = LIB_PATH
+        LIB_PATH = path
+        _lib = None
+        lib()
+    return before
 
 
 def ctr_strerror(code: int) -> str:
@@ -280,3 +295,7 @@ def ctr_goodput(sim_cfg, trace: dict, n_replicas: int, rows_per_replica: int, n_
 
 def ctr_abi_version() -> int:
     return int(lib().ctr_abi_version())
+
+
+def ctr_bounds_checked() -> int:
+    return int(lib().ctr_bounds_checked())

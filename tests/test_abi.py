@@ -36,7 +36,21 @@ def test_exports_every_declared_function(libctr):
 def test_static_entry_points_run_without_gpu(libctr):
     libctr.ctr_strerror.restype = ctypes.c_char_p
     assert libctr.ctr_strerror(-3).decode().startswith("a fixed-capacity")
-    assert libctr.ctr_abi_version() == 6
+    assert libctr.ctr_strerror(-5).decode().startswith("an index fell outside")
+    assert libctr.ctr_abi_version() == 7
+    assert libctr.ctr_bounds_checked() == 0
+
+
+def test_bounds_checked_library_exports_the_same_entry_points():
+    """libctr_checked.so (the simulator compiled with CTR_BOUNDS_CHECK=1) is the
+    same ABI: every declared function, the same version, and it says it is the
+    checked build."""
+    from paper_2609_16206_gb300 import build
+    L = ctypes.CDLL(build.build(checked=True))
+    for name in declared_functions():
+        assert hasattr(L, name), name
+    assert L.ctr_abi_version() == 7
+    assert L.ctr_bounds_checked() == 1
 
 
 def test_step_budget_bound_checked_on_the_host():

@@ -141,7 +141,7 @@ for _ in range(3000):
             except (OverflowError, TypeError):
                 pass
     trace_call(tcfg, pick([0, 1, 2]), pick([0, 5, (1 << 40) - 3]), pick([0, 3]))
-assert L.ctr_abi_version() == 6
+assert L.ctr_abi_version() == 7
 for code in range(-6, 3):
     assert L.ctr_strerror(code)
 print("seen", sorted(seen))
