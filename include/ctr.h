@@ -281,12 +281,14 @@ int ctr_abi_version(void);
 
 /* ctr_bounds_checked -- 1 in libctr_checked.so, 0 in libctr.so.  Both export
  * the same entry points with the same results.  The checked build compiles the
- * simulator's kernels (sim_kernel and its checksum pass) with a bounds check on
- * every index into the workspace, the trace and the outputs: an index outside
- * its buffer skips the access (a load reads 0) and the row ends with
- * CTR_EBOUNDS in row_status (no fault, no trap).  With valid arguments that
- * status never occurs; the checked build exists to show it on the GPU, where
- * no memory checker runs.  It is slower and not meant for production. */
+ * simulator's event loop and the goodput pass with a bounds check on every
+ * index into the workspace, the trace, the outputs and goodput's shared-memory
+ * tables: an index outside its buffer skips the access (a load reads 0) and the
+ * row reports CTR_EBOUNDS -- in row_status from the simulator, in both met_count
+ * and p99_ttft_us from the goodput pass -- with no fault and no trap.  With
+ * valid arguments that value never occurs; the checked build exists to show it
+ * on the GPU, where no memory checker runs.  It is slower and not meant for
+ * production. */
 int ctr_bounds_checked(void);
 
 #ifdef __cplusplus

@@ -20,6 +20,51 @@ constexpr int64_t kArrivalLimit = int64_t(1) << 39;
 constexpr int kKeyBits = 23;                        // request index bits in packed heap keys
 constexpr uint64_t kKeyMask = (uint64_t(1) << kKeyBits) - 1;
 
+// Checked accesses.  A build with CTR_BOUNDS_CHECK=1 compares every index with
+// the length of its buffer first; an index outside skips the access (a load
+// gives 0) and sets `bad`, and the kernel reports CTR_EBOUNDS for the row.
+// Other builds compile the plain access (the length and the flag are dead code
+// there).
+#if CTR_BOUNDS_CHECK
+__device__ __forceinline__ bool ck_out(int64_t i, int64_t len, bool& bad)
+{
+    const bool out = (uint64_t)i >= (uint64_t)len;
+    bad = bad || out;
+    return out;
+}
+#define CTR_CK_OUT(i, len, bad) ck_out((int64_t)(i), (len), (bad))
+#else
+#define CTR_CK_OUT(i, len, bad) false
+#endif
+// true when index i lies in [0, len) (always, in unchecked builds)
+__device__ __forceinline__ bool ck_ok(int64_t i, int64_t len, bool& bad) { return !CTR_CK_OUT(i, len, bad); }
+// (the index keeps the caller's type, so the unchecked address arithmetic is the plain one)
+template <typename T, typename I>
+__device__ __forceinline__ T ck_ld(const T* p, I i, int64_t len, bool& bad)
+{
+    if (CTR_CK_OUT(i, len, bad)) return T();
+    return p[i];
+}
+template <typename T, typename I>
+__device__ __forceinline__ T ck_ldg(const T* p, I i, int64_t len, bool& bad)  // read-only data
+{
+    if (CTR_CK_OUT(i, len, bad)) return T();
+    return __ldg(p + i);
+}
+template <typename T, typename I>
+__device__ __forceinline__ void ck_st(T* p, I i, int64_t len, T v, bool& bad)
+{
+    if (CTR_CK_OUT(i, len, bad)) return;
+    p[i] = v;
+}
+// entries i and i + 1 (i even) as one 16-byte word
+template <typename I>
+__device__ __forceinline__ ulonglong2 ck_ld2(const uint64_t* p, I i, int64_t len, bool& bad)
+{
+    if (CTR_CK_OUT(i, len - 1, bad)) return make_ulonglong2(0, 0);
+    return *reinterpret_cast<const ulonglong2*>(p + i);
+}
+
 // Row checksum term mix(k, tag, v) = sm(sm((tag << 56) ^ k) ^ v), sm the
 // splitmix64 output function (Steele, Lea and Flood, OOPSLA'14).
 __device__ __forceinline__ uint64_t mix64(uint64_t z)

@@ -110,9 +110,20 @@ struct SelScratch {
 // One row's P99 TTFT (and its met count, already reduced) into P.p99 / P.met:
 // from its histogram and staged bins when `staged`, else by the radix select
 // over the TTFTs in global memory (which reuses `hist`).  Block-collective.
+#if CTR_BOUNDS_CHECK
+#define CTR_CK_FLAG_PARAM , bool& bad
+#define CTR_CK_FLAG_ARG , bad
+#else  // the plain build's function keeps its plain signature
+#define CTR_CK_FLAG_PARAM
+#define CTR_CK_FLAG_ARG
+#endif
 __device__ void select_row(const GoodputParams& P, int64_t row, int64_t tb, int64_t n, int32_t met, bool staged,
-                           uint32_t* hist, const uint16_t* bins, SelScratch& S)
+                           uint32_t* hist, const uint16_t* bins, SelScratch& S CTR_CK_FLAG_PARAM)
 {
+#if !CTR_BOUNDS_CHECK
+    bool bad = false;  // dead: the accessors below compile to plain accesses
+#endif
+    const int64_t trace_len = (P.n_rows / P.rows_per_replica) * n, out_len = P.n_rows * n;
     const int tid = threadIdx.x;
     const int64_t ob = row * n;
     const int64_t rank = (99 * n + 99) / 100 - 1;  // 0-based nearest rank
@@ -122,7 +133,7 @@ __device__ void select_row(const GoodputParams& P, int64_t row, int64_t tb, int6
         const uint32_t B = S.pick[0];
         const int64_t r_in = rank - (int64_t)S.pick[1];  // rank among the bin's requests
         for (int64_t k = tid; k < n; k += kThreads) {
-            if (bins[k] == B) {
+            if (ck_ld(bins, k, n, bad) == B) {
                 const uint32_t i = atomicAdd(&S.n_cand, 1u);
                 if (i < (uint32_t)kCand) S.cand_k[i] = (int32_t)k;
             }
@@ -132,7 +143,7 @@ __device__ void select_row(const GoodputParams& P, int64_t row, int64_t tb, int6
         if (c <= kCand) {
             for (int i = tid; i < c; i += kThreads) {
                 const int64_t k = S.cand_k[i];
-                S.cand_v[i] = P.t_first[ob + k] - P.trace.arrival_us[tb + k];
+                S.cand_v[i] = ck_ld(P.t_first, ob + k, out_len, bad) - ck_ld(P.trace.arrival_us, tb + k, trace_len, bad);
             }
             __syncthreads();
             // the candidate whose position in (value, slot) order is the remaining rank
@@ -153,7 +164,7 @@ __device__ void select_row(const GoodputParams& P, int64_t row, int64_t tb, int6
     // ---- fallback: exact radix select over (TTFT - min) read from global memory
     int64_t mn = INT64_MAX, mx = INT64_MIN;
     for (int64_t k = tid; k < n; k += kThreads) {
-        const int64_t t = P.t_first[ob + k] - P.trace.arrival_us[tb + k];
+        const int64_t t = ck_ld(P.t_first, ob + k, out_len, bad) - ck_ld(P.trace.arrival_us, tb + k, trace_len, bad);
         mn = t < mn ? t : mn;
         mx = t > mx ? t : mx;
     }
@@ -171,9 +182,13 @@ __device__ void select_row(const GoodputParams& P, int64_t row, int64_t tb, int6
         __syncthreads();
         const uint32_t dmask = (1u << dbits) - 1u;
         for (int64_t k = tid; k < n; k += kThreads) {
-            const uint64_t v = (uint64_t)(P.t_first[ob + k] - P.trace.arrival_us[tb + k]) - (uint64_t)mn;
+            const uint64_t v = (uint64_t)(ck_ld(P.t_first, ob + k, out_len, bad) -
+                                          ck_ld(P.trace.arrival_us, tb + k, trace_len, bad)) - (uint64_t)mn;
             const bool match = above >= 64 || (v >> above) == (prefix >> above);
-            if (match) atomicAdd(&hist[(uint32_t)(v >> shift) & dmask], 1u);
+            if (match) {
+                const uint32_t b = (uint32_t)(v >> shift) & dmask;
+                if (ck_ok(b, kBins, bad)) atomicAdd(&hist[b], 1u);
+            }
         }
         __syncthreads();
         find_rank_bin(hist, kBins, rk, S.pick, S.wsum);
@@ -199,6 +214,7 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
     const int64_t rpr = P.rows_per_replica;
     const int64_t upr = (rpr + kRows - 1) / kRows;  // units per replica
     const int64_t n_units = (P.n_rows / rpr) * upr;
+    const int64_t trace_len = (P.n_rows / rpr) * n, out_len = P.n_rows * n;  // entries of the trace and outputs
 
     for (int64_t unit = blockIdx.x; unit < n_units; unit += gridDim.x) {
         const int64_t rep = unit / upr;
@@ -218,17 +234,18 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
             h[r] = 0;
         }
         uint32_t wide = 0;  // bit r: row r has a TTFT outside [0, 2^32)
+        bool bad = false;   // bounds-checked builds: an index of this thread fell outside its buffer
         for (int64_t k = tid; k < n; k += kThreads) {
             // every load of the request issued before any is used
-            const int64_t ta = __ldg(&P.trace.arrival_us[tb + k]);
-            const int64_t o = __ldg(&P.trace.true_out[tb + k]);
-            int c = (int)__ldg(&P.trace.slo_class[tb + k]);
+            const int64_t ta = ck_ldg(P.trace.arrival_us, tb + k, trace_len, bad);
+            const int64_t o = ck_ldg(P.trace.true_out, tb + k, trace_len, bad);
+            int c = (int)ck_ldg(P.trace.slo_class, tb + k, trace_len, bad);
             int64_t tf[kRows], td[kRows];
 #pragma unroll
             for (int r = 0; r < kRows; ++r) {
                 if (r < nr) {
-                    tf[r] = __ldg(&P.t_first[(row0 + r) * n + k]);
-                    td[r] = __ldg(&P.t_done[(row0 + r) * n + k]);
+                    tf[r] = ck_ldg(P.t_first, (row0 + r) * n + k, out_len, bad);
+                    td[r] = ck_ldg(P.t_done, (row0 + r) * n + k, out_len, bad);
                 }
             }
             if (c >= P.n_classes) c = P.n_classes - 1;
@@ -236,8 +253,8 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
             uint64_t m2 = 0, m3 = 0;  // the request-only halves of the checksum terms
             if (kHash) {
                 if (P.kmix) {  // mixed once per call (launch_mix_table)
-                    m2 = __ldg(&P.kmix[k]);
-                    m3 = __ldg(&P.kmix[n + k]);
+                    m2 = ck_ldg(P.kmix, k, 2 * n, bad);
+                    m3 = ck_ldg(P.kmix, n + k, 2 * n, bad);
                 } else {
                     m2 = mix64((uint64_t(2) << 56) ^ (uint64_t)k);
                     m3 = mix64((uint64_t(3) << 56) ^ (uint64_t)k);
@@ -252,8 +269,8 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
                     wide |= (uint32_t)!fits << r;
                     if (kStage) {
                         const uint32_t b = fits ? log_bin((uint32_t)ttft) : 0u;
-                        atomicAdd(&hist[r][b], 1u);
-                        bin_s[(int64_t)r * n + k] = (uint16_t)b;
+                        if (ck_ok(b, kLogBins, bad)) atomicAdd(&hist[r][b], 1u);
+                        ck_st(bin_s, (int64_t)r * n + k, (int64_t)kRows * n, (uint16_t)b, bad);
                     }
                     if (kHash) h[r] += mix64(m2 ^ (uint64_t)tf[r]) + mix64(m3 ^ (uint64_t)td[r]);
                 }
@@ -280,7 +297,14 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
                     }
                     continue;
                 }
-                select_row(P, row, tb, n, m_r, kStage && !((wide >> r) & 1u), hist[r], bin_s + (int64_t)r * n, S);
+                select_row(P, row, tb, n, m_r, kStage && !((wide >> r) & 1u), hist[r], bin_s + (int64_t)r * n,
+                           S CTR_CK_FLAG_ARG);
+#if CTR_BOUNDS_CHECK
+                if (__syncthreads_or(bad) && tid == 0) {  // a row whose pass left a buffer: both outputs say so
+                    P.met[row] = CTR_EBOUNDS;
+                    P.p99[row] = CTR_EBOUNDS;
+                }
+#endif
             }
         }
     }

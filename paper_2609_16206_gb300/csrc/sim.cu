@@ -112,48 +112,6 @@ __device__ __forceinline__ int64_t kv_term(int64_t x, const SimParams& P)
     return (int64_t)((hi + (lo >> 32)) >> 32);  // no overflow: hi <= 2^64 - 2^33 + 1
 }
 
-// Checked accesses.  A build with CTR_BOUNDS_CHECK=1 compares every index with
-// the length of its buffer first; an index outside skips the access (a load
-// gives 0) and sets `bad`, and the row ends with CTR_EBOUNDS.  Other builds
-// compile the plain access (the length and the flag are dead code there).
-#if CTR_BOUNDS_CHECK
-__device__ __forceinline__ bool ck_out(int64_t i, int64_t len, bool& bad)
-{
-    const bool out = (uint64_t)i >= (uint64_t)len;
-    bad = bad || out;
-    return out;
-}
-#define CTR_CK_OUT(i, len, bad) ck_out((int64_t)(i), (len), (bad))
-#else
-#define CTR_CK_OUT(i, len, bad) false
-#endif
-// (the index keeps the caller's type, so the unchecked address arithmetic is the plain one)
-template <typename T, typename I>
-__device__ __forceinline__ T ck_ld(const T* p, I i, int64_t len, bool& bad)
-{
-    if (CTR_CK_OUT(i, len, bad)) return T();
-    return p[i];
-}
-template <typename T, typename I>
-__device__ __forceinline__ T ck_ldg(const T* p, I i, int64_t len, bool& bad)  // read-only data
-{
-    if (CTR_CK_OUT(i, len, bad)) return T();
-    return __ldg(p + i);
-}
-template <typename T, typename I>
-__device__ __forceinline__ void ck_st(T* p, I i, int64_t len, T v, bool& bad)
-{
-    if (CTR_CK_OUT(i, len, bad)) return;
-    p[i] = v;
-}
-// entries i and i + 1 (i even) as one 16-byte word
-template <typename I>
-__device__ __forceinline__ ulonglong2 ck_ld2(const uint64_t* p, I i, int64_t len, bool& bad)
-{
-    if (CTR_CK_OUT(i, len - 1, bad)) return make_ulonglong2(0, 0);
-    return *reinterpret_cast<const ulonglong2*>(p + i);
-}
-
 // Entries per lane of a heap region holding up to cap keys.  The heaps are
 // 4-ary: node j (0-based) sits at position j + 3, so its children 4j + 1 ..
 // 4j + 4 sit at positions 4j + 4 .. 4j + 7, a 32-byte aligned block read as

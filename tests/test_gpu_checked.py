@@ -1,17 +1,20 @@
-"""The simulator's parity cases again, on libctr_checked.so: the same kernels
-compiled with CTR_BOUNDS_CHECK=1, so that every index into the workspace
-(heaps, rings, FIFOs), the trace and the outputs is compared with its buffer's
-length before the access.  An index outside would skip the access and end its
-row with CTR_EBOUNDS, which no oracle status equals, so each case below passes
-only if no access of the run left its buffer.  This is the device-side memory
-check where no memory checker runs: tiny capacities (every overflow path),
-every pool width, batched prefill, the proxy's signals, random configurations
-and the benchmarked launch itself."""
+"""The simulator's and the goodput pass's parity cases again, on
+libctr_checked.so: the same kernels compiled with CTR_BOUNDS_CHECK=1, so that
+every index into the workspace (heaps, rings, FIFOs), the trace, the outputs
+and goodput's shared histograms, staged bins and P99 candidates is compared
+with its buffer's length before the access.  An index outside would skip the
+access and end its row with CTR_EBOUNDS (in the simulator's status, in
+goodput's met count and P99), which no oracle value equals, so each case below
+passes only if no access of the run left its buffer.  This is the device-side
+memory check where no memory checker runs: tiny capacities (every overflow
+path), every pool width, batched prefill, the proxy's signals, random
+configurations, adversarial and crowded TTFTs, and the benchmarked launch."""
 import pytest
 import torch
 
 import simutil as U
 import test_gpu_fuzz as F
+import test_gpu_goodput as G
 import test_gpu_sim as S
 from gpuutil import need_gpu
 from paper_2609_16206_gb300 import workloads as W
@@ -87,6 +90,28 @@ def test_batched_prefill_document(orc, budget):
 @pytest.mark.parametrize("seed", range(0, 160, 4))
 def test_random_configuration(orc, seed):
     F.test_random_configuration(orc, seed)
+
+
+@pytest.mark.parametrize("wl,R,N", [(W.replica_sweep(), 8, 5000), (W.large_pool(rate_mreq=34_000), 2, 3000),
+                                    (W.replica_sweep(), 3, 37), (W.replica_sweep(), 1, 45_000)],
+                         ids=["2p6d", "4p28d", "short", "unstaged"])
+def test_goodput(orc, wl, R, N):
+    G.test_goodput_matches_oracle(orc, wl, R, N)
+
+
+def test_goodput_adversarial_times(orc):
+    G.test_goodput_adversarial_times(orc)
+
+
+@pytest.mark.parametrize("crowd", [1, 512, 513, 3000])
+def test_goodput_crowded_p99_bin(orc, crowd):
+    G.test_goodput_crowded_p99_bin(orc, crowd)
+
+
+@pytest.mark.parametrize("wl,R,N,sets", [(W.replica_sweep(), 6, 4000, 1), (W.replica_sweep(), 3, 45_000, 1)],
+                         ids=["staged", "unstaged"])
+def test_goodput_inside_simulate(orc, wl, R, N, sets):
+    G.test_goodput_inside_simulate_matches_the_standalone_call(orc, wl, R, N, sets)
 
 
 def test_benchmarked_launch(orc):
