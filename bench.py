@@ -593,7 +593,8 @@ def run_ours(args, rank, world, local_rank):
                          "the place of on-device trace generation (ctr_gen_trace), so this step does that much "
                          "less device work than the device-timed step",
                  "steps": e2e_steps},
-        "gpu_launches": 4 * args.steps,  # trace, simulation, checksum + goodput pass, scorer
+        # per step: trace, simulation, the checksum's request-only mix table, checksum + goodput pass, scorer
+        "gpu_launches": 5 * args.steps,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)
