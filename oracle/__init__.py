@@ -113,6 +113,8 @@ def lib():
             L.orc_goodput.argtypes = [C.POINTER(_SimCfg), C.c_int64, C.POINTER(C.c_int64), C.POINTER(C.c_int32),
                                       C.POINTER(C.c_uint8), C.POINTER(C.c_int64), C.POINTER(C.c_int64),
                                       C.POINTER(C.c_int64), C.POINTER(C.c_int64)]
+            L.orc_p99_tpot.argtypes = [C.c_int64, C.POINTER(C.c_int32), C.POINTER(C.c_int64), C.POINTER(C.c_int64),
+                                       C.POINTER(C.c_int64)]
             L.orc_score_batch.argtypes = [C.POINTER(C.c_float), C.POINTER(C.c_float), C.POINTER(C.c_uint8),
                                           C.c_int64, C.POINTER(C.c_float), C.POINTER(C.c_float),
                                           C.POINTER(C.c_float), C.c_int64, C.POINTER(C.c_float),
@@ -293,6 +295,18 @@ def goodput(sc, trace: dict, t_first, t_done):
     if rc != OK:
         raise RuntimeError(f"orc_goodput failed: {rc}")
     return int(met.value), int(p99.value)
+
+
+def p99_tpot(trace: dict, t_first, t_done) -> int:
+    """Nearest-rank P99 of floor((t_done - t_first) / (o - 1)) over one row's requests with o >= 2 (-1: none)."""
+    o = np.ascontiguousarray(trace["true_out"], np.int32)
+    tf = np.ascontiguousarray(t_first, np.int64)
+    td = np.ascontiguousarray(t_done, np.int64)
+    out = C.c_int64(0)
+    rc = lib().orc_p99_tpot(o.size, _p(o, C.c_int32), _p(tf, C.c_int64), _p(td, C.c_int64), C.byref(out))
+    if rc != OK:
+        raise RuntimeError(f"orc_p99_tpot failed: {rc}")
+    return int(out.value)
 
 
 # ---------------------------------------------------------------- scorer

@@ -23,7 +23,7 @@
  *     binary heap of events.  Per-instance aggregates (queue length,
  *     remaining work, resident KV) are recomputed from per-request state
  *     by scanning, never kept as running counters.
- *   - SLO goodput and nearest-rank P99 TTFT (sec. IV-B, Table 2) by sorting.
+ *   - SLO goodput and nearest-rank P99 TTFT and TPOT (sec. IV-B, Table 2) by sorting.
  *   - The standalone fp64 brute-force request x instance scorer.
  *
  * Every function names the passage it follows.  Where the paper is silent
@@ -1000,6 +1000,31 @@ int orc_goodput(const orc_sim_cfg* cfg, int64_t n, const int64_t* arr, const int
     *met_out = met;
     *p99_out = ttft[(99 * n + 99) / 100 - 1];
     free(ttft);
+    return ORC_OK;
+}
+
+/* ======================================================================
+ * P99 TPOT of one row (Table 2's third column; sec. IV-B names TPOT targets).
+ * [reading] A request's time per output token counts the tokens after its
+ * first: TPOT = floor((t_done - t_first) / (o - 1)) us for o >= 2; a request of
+ * one output token has none.  The row's P99 is the nearest rank, sorted index
+ * ceil(0.99 M) - 1, over its M requests with o >= 2; M = 0 gives -1.
+ * ==================================================================== */
+int orc_p99_tpot(int64_t n, const int32_t* o, const int64_t* t_first, const int64_t* t_done, int64_t* p99_out)
+{
+    *p99_out = -1;
+    if (n <= 0) return ORC_OK;
+    int64_t* tpot = (int64_t*)malloc((size_t)n * 8);
+    if (!tpot) return ORC_ENOMEM;
+    int64_t m = 0;
+    for (int64_t k = 0; k < n; ++k) {
+        if (o[k] >= 2) tpot[m++] = (t_done[k] - t_first[k]) / ((int64_t)o[k] - 1);
+    }
+    if (m > 0) {
+        qsort(tpot, (size_t)m, 8, cmp_i64);
+        *p99_out = tpot[(99 * m + 99) / 100 - 1];
+    }
+    free(tpot);
     return ORC_OK;
 }
 
