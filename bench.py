@@ -607,17 +607,17 @@ def run_ours(args, rank, world, local_rank):
 # per routed request, keyed by a hash of the simulator's code: a stale entry
 # (the kernel changed since the counters were taken) reports null.
 SIM_SLICE_COUNTERS: dict = {
-    "74c2a52e0a4a5664": {"warp_inst_per_routed": 34162633267 / 81_920_000,
+    "19c8159da076dbe6": {"warp_inst_per_routed": 34162633267 / 81_920_000,
                          "thread_inst_per_warp_inst": 281165931678 / 34162633267,
-                         "dram_bytes_per_routed": (2387567360 + 1565587712) / 81_920_000,
+                         "dram_bytes_per_routed": (2387482368 + 1564797184) / 81_920_000,
                          "slice": "ncu on one launch of 1,024 replicas x 20,000 requests x 4 policies "
                                   "(81.92 M routed requests): 3.416e10 warp-instructions, 2.812e11 thread-"
-                                  "instructions, 2.388 GB DRAM read + 1.566 GB written"},
+                                  "instructions, 2.387 GB DRAM read + 1.565 GB written"},
 }
 
 # DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.
 SCORE_DRAM_PER_LAUNCH: dict = {
-    "17e84ac0f5668c9d": {"read": 9486080.0, "write": 0.0},
+    "027701a27e0c2fcd": {"read": 9484800.0, "write": 0.0},
 }
 
 

@@ -267,10 +267,14 @@ int ctr_simulate_noalloc(const ctr_sim_cfg* cfg /* host */, const ctr_cost_const
  * t_done - t_first <= TPOT_c (o - 1))} and p99_ttft_us[row] = the nearest-rank
  * P99 (sorted index ceil(0.99 n) - 1; -1 when n_req == 0).  Row r uses replica
  * r / rows_per_replica of the trace.  A class >= n_classes counts as the last
- * class. */
+ * class.
+ * p99_tpot_us: optional (NULL: not computed).  Table 2's P99 TPOT: over the
+ * row's M requests with o >= 2, each one's (t_done - t_first) / (o - 1)
+ * rounded toward zero, the nearest-rank P99 (sorted index ceil(0.99 M) - 1;
+ * -1 when M == 0), computed in a pass of its own after the goodput pass. */
 int ctr_goodput(const ctr_sim_cfg* cfg /* host */, ctr_requests trace, int32_t n_replicas, int32_t rows_per_replica,
                 int64_t n_req, const int64_t* t_first_us, const int64_t* t_done_us, int64_t* met_count,
-                int64_t* p99_ttft_us, void* stream);
+                int64_t* p99_ttft_us, int64_t* p99_tpot_us, void* stream);
 
 /* ctr_strerror -- static description of a CTR_* code. */
 const char* ctr_strerror(int code);

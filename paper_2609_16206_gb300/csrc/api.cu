@@ -10,7 +10,7 @@ using namespace ctr;
 
 namespace {
 
-constexpr int kAbiVersion = 7;
+constexpr int kAbiVersion = 8;
 
 bool in_range(int64_t v, int64_t lo, int64_t hi) { return v >= lo && v <= hi; }
 
@@ -346,7 +346,7 @@ int ctr_simulate(const ctr_sim_cfg* cfg, const ctr_cost_consts* consts, int32_t 
 
 int ctr_goodput(const ctr_sim_cfg* cfg, ctr_requests trace, int32_t n_replicas, int32_t rows_per_replica, int64_t n_req,
                 const int64_t* t_first_us, const int64_t* t_done_us, int64_t* met_count, int64_t* p99_ttft_us,
-                void* stream)
+                int64_t* p99_tpot_us, void* stream)
 {
     if (!cfg || !in_range(cfg->n_classes, 1, CTR_MAX_CLASSES)) return CTR_EINVAL;
     if (n_replicas < 0 || rows_per_replica < 1 || !in_range(n_req, 0, CTR_MAX_REQUESTS)) return CTR_EINVAL;
@@ -369,7 +369,9 @@ int ctr_goodput(const ctr_sim_cfg* cfg, ctr_requests trace, int32_t n_replicas, 
     p.t_done = t_done_us;
     p.met = met_count;
     p.p99 = p99_ttft_us;
-    return cuda_status(launch_goodput(p, (cudaStream_t)stream));
+    const cudaError_t e = launch_goodput(p, (cudaStream_t)stream);
+    if (e != cudaSuccess || !p99_tpot_us) return cuda_status(e);
+    return cuda_status(launch_tpot(p, p99_tpot_us, (cudaStream_t)stream));
 }
 
 }  // extern "C"

@@ -197,6 +197,8 @@ struct GoodputParams {
     const uint64_t* kmix;  // optional with row_hash: the table of launch_mix_table for n_req
 };
 cudaError_t launch_goodput(const GoodputParams& p, cudaStream_t stream);
+// Each row's nearest-rank P99 TPOT into p99_tpot[row] (-1 when no request has two tokens or more).
+cudaError_t launch_tpot(const GoodputParams& p, int64_t* p99_tpot, cudaStream_t stream);
 
 // ---------------------------------------------------------------- standalone scorer
 struct ScoreParams {

@@ -1,6 +1,7 @@
 // goodput.cu -- SLO goodput inputs per simulated row (ctr_goodput):
 // the count of requests meeting both SLOs of their class (sec. IV-B targets,
-// Table 2 goodput) and the exact nearest-rank P99 TTFT (Table 2 column).
+// Table 2 goodput), the exact nearest-rank P99 TTFT and, on request, the
+// exact nearest-rank P99 TPOT (Table 2 columns; tpot_kernel at the end).
 //
 // One block per unit of up to kRows rows of one replica, which share the
 // replica's trace and request indices.  Pass 0 reads the unit once: per
@@ -310,6 +311,131 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
     }
 }
 
+// P99 TPOT per row (Table 2): one block per row.  A request with o >= 2
+// output tokens has TPOT = (t_done - t_first) / (o - 1) rounded toward zero
+// (the floor, as t_done >= t_first); one-token requests have none.  Pass 1
+// counts the row's M such requests and histograms their TPOTs over the same
+// logarithmic bins as the TTFTs (32-bit quotients when the decode time is
+// below 2^32 us); a block scan finds the bin of the nearest rank
+// ceil(0.99 M) - 1; pass 2 gathers that bin's TPOTs and counts the remaining
+// rank out exactly.  A decode time outside [0, 2^32) or more than kCand
+// requests in the bin fall back to an exact radix select (11-bit digits) over
+// the 64-bit quotients.
+__device__ __forceinline__ bool tpot_of(const GoodputParams& P, int64_t tb, int64_t ob, int64_t k, int64_t& v)
+{
+    const int32_t o = __ldg(&P.trace.true_out[tb + k]);
+    if (o < 2) return false;
+    v = (__ldg(&P.t_done[ob + k]) - __ldg(&P.t_first[ob + k])) / (int64_t)(o - 1);
+    return true;
+}
+// the same for a row whose decode times all lie in [0, 2^32): one 32-bit quotient
+__device__ __forceinline__ bool tpot32_of(const GoodputParams& P, int64_t tb, int64_t ob, int64_t k, uint32_t& v)
+{
+    const int32_t o = __ldg(&P.trace.true_out[tb + k]);
+    if (o < 2) return false;
+    v = (uint32_t)(__ldg(&P.t_done[ob + k]) - __ldg(&P.t_first[ob + k])) / (uint32_t)(o - 1);
+    return true;
+}
+
+__global__ void __launch_bounds__(kThreads, 2) tpot_kernel(const GoodputParams P, int64_t* p99_tpot)
+{
+    __shared__ uint32_t hist[kLogBins];
+    __shared__ SelScratch S;
+    const int tid = threadIdx.x;
+    const int64_t n = P.n_req;
+    for (int64_t row = blockIdx.x; row < P.n_rows; row += gridDim.x) {
+        const int64_t tb = (row / P.rows_per_replica) * n, ob = row * n;
+        for (int i = tid; i < kLogBins; i += kThreads) hist[i] = 0;
+        __syncthreads();
+        int32_t m = 0;
+        int32_t wide = 0;  // a decode time outside [0, 2^32)
+        for (int64_t k = tid; k < n; k += kThreads) {
+            const int32_t o = __ldg(&P.trace.true_out[tb + k]);
+            if (o < 2) continue;
+            m += 1;
+            const int64_t d = __ldg(&P.t_done[ob + k]) - __ldg(&P.t_first[ob + k]);
+            if ((uint64_t)d < (uint64_t(1) << 32)) {
+                atomicAdd(&hist[log_bin((uint32_t)d / (uint32_t)(o - 1))], 1u);
+            } else {
+                wide = 1;
+            }
+        }
+        const int32_t M = block_reduce<int32_t>(m, 0, [](int32_t a, int32_t b) { return a + b; },
+                                                reinterpret_cast<int32_t*>(S.red64));
+        wide = block_reduce<int32_t>(wide, 0, [](int32_t a, int32_t b) { return a | b; },
+                                     reinterpret_cast<int32_t*>(S.red64));
+        if (M == 0) {
+            if (tid == 0) p99_tpot[row] = -1;
+            continue;
+        }
+        const int64_t rank = (99 * (int64_t)M + 99) / 100 - 1;  // 0-based nearest rank among the M
+        if (!wide) {
+            if (tid == 0) S.n_cand = 0;
+            find_rank_bin(hist, kLogBins, rank, S.pick, S.wsum);  // its barriers also publish n_cand
+            const uint32_t B = S.pick[0];
+            const int64_t r_in = rank - (int64_t)S.pick[1];
+            for (int64_t k = tid; k < n; k += kThreads) {
+                uint32_t v;
+                if (tpot32_of(P, tb, ob, k, v) && log_bin(v) == B) {
+                    const uint32_t i = atomicAdd(&S.n_cand, 1u);
+                    if (i < (uint32_t)kCand) S.cand_v[i] = (int64_t)v;
+                }
+            }
+            __syncthreads();
+            const int c = (int)S.n_cand;
+            if (c <= kCand) {
+                for (int i = tid; i < c; i += kThreads) {
+                    const int64_t v = S.cand_v[i];
+                    int64_t pos = 0;
+                    for (int j = 0; j < c; ++j) {
+                        const int64_t w = S.cand_v[j];
+                        pos += w < v || (w == v && j < i);
+                    }
+                    if (pos == r_in) p99_tpot[row] = v;
+                }
+                __syncthreads();
+                continue;
+            }
+        }
+        // exact radix select over (TPOT - min) of the row's multi-token requests
+        int64_t mn = INT64_MAX, mx = INT64_MIN;
+        for (int64_t k = tid; k < n; k += kThreads) {
+            int64_t v;
+            if (tpot_of(P, tb, ob, k, v)) {
+                mn = v < mn ? v : mn;
+                mx = v > mx ? v : mx;
+            }
+        }
+        mn = block_reduce<int64_t>(mn, INT64_MAX, [](int64_t a, int64_t b) { return a < b ? a : b; }, S.red64);
+        mx = block_reduce<int64_t>(mx, INT64_MIN, [](int64_t a, int64_t b) { return a > b ? a : b; }, S.red64);
+        const uint64_t range = (uint64_t)mx - (uint64_t)mn;
+        int shift = range == 0 ? 0 : 64 - __clzll((long long)range);
+        uint64_t prefix = 0;
+        int64_t rk = rank;
+        while (shift > 0) {
+            const int dbits = shift < kDigit ? shift : kDigit;
+            const int above = shift;
+            shift -= dbits;
+            for (int i = tid; i < kBins; i += kThreads) hist[i] = 0;
+            __syncthreads();
+            const uint32_t dmask = (1u << dbits) - 1u;
+            for (int64_t k = tid; k < n; k += kThreads) {
+                int64_t tv;
+                if (!tpot_of(P, tb, ob, k, tv)) continue;
+                const uint64_t v = (uint64_t)tv - (uint64_t)mn;
+                if (above >= 64 || (v >> above) == (prefix >> above)) atomicAdd(&hist[(uint32_t)(v >> shift) & dmask], 1u);
+            }
+            __syncthreads();
+            find_rank_bin(hist, kBins, rk, S.pick, S.wsum);
+            prefix |= (uint64_t)S.pick[0] << shift;
+            rk -= S.pick[1];
+            __syncthreads();
+        }
+        if (tid == 0) p99_tpot[row] = (int64_t)((uint64_t)mn + prefix);
+        __syncthreads();
+    }
+}
+
 __global__ void __launch_bounds__(256) mix_table_kernel(uint64_t* t, int64_t n)
 {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < 2 * n; i += (int64_t)gridDim.x * blockDim.x) {
@@ -341,6 +467,19 @@ cudaError_t launch_rows(const GoodputParams& p, int64_t dyn_bytes, bool hash, in
 }
 
 }  // namespace
+
+cudaError_t launch_tpot(const GoodputParams& p, int64_t* p99_tpot, cudaStream_t stream)
+{
+    if (p.n_rows == 0) return cudaSuccess;
+    int dev = 0, sms = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    const int64_t blocks = p.n_rows < (int64_t)sms * 2 ? p.n_rows : (int64_t)sms * 2;
+    tpot_kernel<<<(unsigned)blocks, kThreads, 0, stream>>>(p, p99_tpot);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_mix_table(uint64_t* t, int64_t n, cudaStream_t stream)
 {

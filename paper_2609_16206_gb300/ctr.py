@@ -102,7 +102,7 @@ def lib():
             L.ctr_simulate_noalloc.argtypes = [C.POINTER(CtrSimCfg), C.POINTER(CtrCostConsts), i32, C.POINTER(i32),
                                                i32, CtrRequests, i32, i64, vp, vp, vp, vp, vp, vp, vp]
             L.ctr_simulate_noalloc.restype = C.c_int
-            L.ctr_goodput.argtypes = [C.POINTER(CtrSimCfg), CtrRequests, i32, i32, i64, vp, vp, vp, vp, vp]
+            L.ctr_goodput.argtypes = [C.POINTER(CtrSimCfg), CtrRequests, i32, i32, i64, vp, vp, vp, vp, vp, vp]
             L.ctr_goodput.restype = C.c_int
             L.ctr_strerror.argtypes = [C.c_int]
             L.ctr_strerror.restype = C.c_char_p
@@ -286,11 +286,11 @@ def ctr_simulate_noalloc(sim_cfg, const_sets, policies, trace: dict, n_replicas:
 
 
 def ctr_goodput(sim_cfg, trace: dict, n_replicas: int, rows_per_replica: int, n_req: int, t_first_us, t_done_us,
-                met_count, p99_ttft_us, stream=None):
+                met_count, p99_ttft_us, p99_tpot_us=None, stream=None):
     cfg = sim_cfg_struct(sim_cfg)
     _check("ctr_goodput", lib().ctr_goodput(
         C.byref(cfg), requests_struct(trace), int(n_replicas), int(rows_per_replica), int(n_req), _ptr(t_first_us),
-        _ptr(t_done_us), _ptr(met_count), _ptr(p99_ttft_us), _stream(stream)))
+        _ptr(t_done_us), _ptr(met_count), _ptr(p99_ttft_us), _ptr(p99_tpot_us), _stream(stream)))
 
 
 def ctr_abi_version() -> int:

@@ -37,7 +37,7 @@ def test_static_entry_points_run_without_gpu(libctr):
     libctr.ctr_strerror.restype = ctypes.c_char_p
     assert libctr.ctr_strerror(-3).decode().startswith("a fixed-capacity")
     assert libctr.ctr_strerror(-5).decode().startswith("an index fell outside")
-    assert libctr.ctr_abi_version() == 7
+    assert libctr.ctr_abi_version() == 8
     assert libctr.ctr_bounds_checked() == 0
 
 
@@ -49,7 +49,7 @@ def test_bounds_checked_library_exports_the_same_entry_points():
     L = ctypes.CDLL(build.build(checked=True))
     for name in declared_functions():
         assert hasattr(L, name), name
-    assert L.ctr_abi_version() == 7
+    assert L.ctr_abi_version() == 8
     assert L.ctr_bounds_checked() == 1
 
 
@@ -92,7 +92,7 @@ def test_request_count_bound_checked_on_the_host():
                               None, None, None, None, None, None, 0, None)
 
     def goodput(n_req):
-        return L.ctr_goodput(ctypes.byref(cfg), ctr.CtrRequests(), 0, 4, n_req, None, None, None, None, None)
+        return L.ctr_goodput(ctypes.byref(cfg), ctr.CtrRequests(), 0, 4, n_req, None, None, None, None, None, None)
     assert sim(M) == ctr.CTR_OK and sim(M + 1) == ctr.CTR_EINVAL and sim(-1) == ctr.CTR_EINVAL
     assert goodput(M) == ctr.CTR_OK and goodput(M + 1) == ctr.CTR_EINVAL
     tcfg = ctr.trace_cfg_struct(W.TraceCfg())

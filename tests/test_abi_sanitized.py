@@ -114,8 +114,8 @@ rc(L.ctr_score_batch(None, ptr, ptr, 10, ptr, ptr, ptr, 4, cv, ptr, ptr, None, N
 rc(L.ctr_score_batch(ptr, ptr, ptr, 10, ptr, ptr, ptr, 4, None, ptr, ptr, None, None))
 # goodput
 for n_rep, rows_per, n_req in ((-1, 4, 10), (1, 0, 10), (1, 4, -1), ((1 << 31) - 1, (1 << 31) - 1, 1), (0, 4, 10)):
-    rc(L.ctr_goodput(C.byref(base), req, n_rep, rows_per, n_req, ptr, ptr, ptr, ptr, None))
-rc(L.ctr_goodput(None, req, 1, 4, 10, ptr, ptr, ptr, ptr, None))
+    rc(L.ctr_goodput(C.byref(base), req, n_rep, rows_per, n_req, ptr, ptr, ptr, ptr, None, None))
+rc(L.ctr_goodput(None, req, 1, 4, 10, ptr, ptr, ptr, ptr, None, None))
 # seeded random configurations
 rng = np.random.default_rng(1)
 pick = lambda xs: xs[int(rng.integers(len(xs)))]
@@ -141,7 +141,7 @@ for _ in range(3000):
             except (OverflowError, TypeError):
                 pass
     trace_call(tcfg, pick([0, 1, 2]), pick([0, 5, (1 << 40) - 3]), pick([0, 3]))
-assert L.ctr_abi_version() == 7
+assert L.ctr_abi_version() == 8
 for code in range(-6, 3):
     assert L.ctr_strerror(code)
 print("seen", sorted(seen))

@@ -1,4 +1,4 @@
-"""Parity: GPU goodput (SLO-met count, nearest-rank P99 TTFT) equals the oracle's."""
+"""Parity: GPU goodput (SLO-met count, nearest-rank P99 TTFT and P99 TPOT) equals the oracle's."""
 import numpy as np
 import pytest
 import torch
@@ -147,3 +147,66 @@ def test_goodput_outputs_come_in_pairs():
                                                                                        device="cuda"), ws,
                          met_count=torch.zeros(4, dtype=torch.int64, device="cuda"))
     assert err.value.code == ctr.CTR_EINVAL
+
+
+def _p99_tpot(ctr, sc, tr, R, rows_per, N, tf, td):
+    rows = R * rows_per
+    met = torch.empty(rows, dtype=torch.int64, device="cuda")
+    p99 = torch.empty(rows, dtype=torch.int64, device="cuda")
+    tpot = torch.full((rows,), -5, dtype=torch.int64, device="cuda")
+    ctr.ctr_goodput(sc, tr, R, rows_per, N, tf, td, met, p99, p99_tpot_us=tpot)
+    torch.cuda.synchronize()
+    return tpot.cpu().numpy()
+
+
+@pytest.mark.parametrize("wl,R,N", [(W.single_replica(), 1, 2000), (W.replica_sweep(), 8, 5000),
+                                    (W.large_pool(rate_mreq=34_000), 2, 3000), (W.replica_sweep(), 3, 37),
+                                    (W.document(rate_mreq=9_000), 2, 3000), (W.replica_sweep(), 1, 45_000)])
+def test_p99_tpot_matches_oracle(orc, wl, R, N):
+    """Table 2's P99 TPOT of every simulated row, bit for bit."""
+    ctr = need_gpu()
+    tr = gen(ctr, wl.trace, R, N)
+    pols = list(W.ALL_POLICIES)
+    res = simulate(ctr, wl.sim, [wl.consts[0]], pols, tr, R, N)
+    tpot = _p99_tpot(ctr, wl.sim, tr, R, len(pols), N, torch.from_numpy(res["t_first_us"]).cuda(),
+                     torch.from_numpy(res["t_done_us"]).cuda())
+    for r in range(R):
+        trh = host_trace(tr, r)
+        for j in range(len(pols)):
+            row = r * len(pols) + j
+            assert tpot[row] == orc.p99_tpot(trh, res["t_first_us"][row], res["t_done_us"][row]), (r, j)
+
+
+@pytest.mark.parametrize("case", ["crowded", "wide", "negative", "one_token", "few", "empty"])
+def test_p99_tpot_adversarial(orc, case):
+    """Crowded bins (over 512 equal TPOTs at the rank), decode times of 2^32 us and more, negative
+    decode times (radix select), rows without a multi-token request (-1), single requests, empty rows."""
+    ctr = need_gpu()
+    rng = np.random.default_rng(len(case))
+    R, N = 3, 6000
+    o = rng.integers(1, 300, (R, N))
+    o[rng.random((R, N)) < 0.2] = 1
+    tf = rng.integers(0, 10**9, (R, N))
+    td = tf + rng.integers(0, 10**7, (R, N))
+    if case == "crowded":
+        td = tf + 30_000 * np.maximum(o - 1, 0) + rng.integers(0, 2, (R, N))  # TPOTs 30,000 or just above
+    elif case == "wide":
+        td[:, 5] = tf[:, 5] + (1 << 33) + 12345
+    elif case == "negative":
+        td[1] = tf[1] - rng.integers(0, 10**6, N)
+    elif case == "one_token":
+        o[:] = 1
+    elif case == "few":
+        o[:] = 1
+        o[0, 17] = 2
+        o[2, :3] = 7
+    elif case == "empty":
+        N = 0
+        o, tf, td = o[:, :0], tf[:, :0], td[:, :0]
+    trh = {"arrival_us": np.sort(rng.integers(0, 10**6, (R, N)), axis=1), "prompt_len": np.ones((R, N)),
+           "true_out": o, "pred_out": np.ones((R, N)), "slo_class": np.zeros((R, N))}
+    tpot = _p99_tpot(ctr, W.SimCfg(), to_dev(trh), R, 1, N, torch.from_numpy(tf).cuda(), torch.from_numpy(td).cuda())
+    for r in range(R):
+        assert tpot[r] == orc.p99_tpot({"true_out": o[r]}, tf[r], td[r]), (case, r)
+    if case in ("one_token", "empty"):
+        assert tpot.tolist() == [-1, -1, -1]
