@@ -591,7 +591,8 @@ def run_ours(args, rank, world, local_rank):
                          "overlaps this step's compute on a second stream, double-buffered), simulate + goodput + "
                          "score, per-row results and scorer outputs copied out; the host copy of the trace takes "
                          "the place of on-device trace generation (ctr_gen_trace), so this step does that much "
-                         "less device work than the device-timed step",
+                         "less device work than the device-timed step; the first step's copy has no compute to "
+                         "overlap (the pipeline fills once per run of e2e steps)",
                  "steps": e2e_steps},
         # per step: trace, simulation, the checksum's request-only mix table, checksum + goodput pass, scorer
         "gpu_launches": 5 * args.steps,
