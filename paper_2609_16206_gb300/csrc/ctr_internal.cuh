@@ -57,11 +57,17 @@ __device__ __forceinline__ void ck_st(T* p, I i, int64_t len, T v, bool& bad)
     if (CTR_CK_OUT(i, len, bad)) return;
     p[i] = v;
 }
-// entries i and i + 1 (i even) as one 16-byte word
+// entries i and i + 1 as one 16-byte word (the checked build also checks its 16-byte alignment)
 template <typename I>
 __device__ __forceinline__ ulonglong2 ck_ld2(const uint64_t* p, I i, int64_t len, bool& bad)
 {
     if (CTR_CK_OUT(i, len - 1, bad)) return make_ulonglong2(0, 0);
+#if CTR_BOUNDS_CHECK
+    if ((reinterpret_cast<uintptr_t>(p + i) & 15u) != 0) {
+        bad = true;
+        return make_ulonglong2(0, 0);
+    }
+#endif
     return *reinterpret_cast<const ulonglong2*>(p + i);
 }
 
