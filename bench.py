@@ -608,17 +608,17 @@ def run_ours(args, rank, world, local_rank):
 # per routed request, keyed by a hash of the simulator's code: a stale entry
 # (the kernel changed since the counters were taken) reports null.
 SIM_SLICE_COUNTERS: dict = {
-    "19c8159da076dbe6": {"warp_inst_per_routed": 34162633267 / 81_920_000,
+    "5b2cb8e0e1f5e9de": {"warp_inst_per_routed": 34162633267 / 81_920_000,
                          "thread_inst_per_warp_inst": 281165931678 / 34162633267,
-                         "dram_bytes_per_routed": (2387482368 + 1564797184) / 81_920_000,
+                         "dram_bytes_per_routed": (2383411200 + 1563864576) / 81_920_000,
                          "slice": "ncu on one launch of 1,024 replicas x 20,000 requests x 4 policies "
                                   "(81.92 M routed requests): 3.416e10 warp-instructions, 2.812e11 thread-"
-                                  "instructions, 2.387 GB DRAM read + 1.565 GB written"},
+                                  "instructions, 2.383 GB DRAM read + 1.564 GB written"},
 }
 
 # DRAM bytes of one scorer launch (2^20 requests x 64 instances) inside the step.
 SCORE_DRAM_PER_LAUNCH: dict = {
-    "027701a27e0c2fcd": {"read": 9484800.0, "write": 0.0},
+    "f16cba77579b1bc7": {"read": 9484800.0, "write": 0.0},
 }
 
 
