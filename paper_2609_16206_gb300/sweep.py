@@ -13,6 +13,9 @@
   pool-width sweep grid and its offered rates.
 * ``noise_sweep`` -- the predictor-noise sweep of sec. V-G: the same replicas
   at every noise level (common random numbers), one simulation call.
+* ``policy_table`` -- Table 2's columns per policy (goodput, P99 TTFT, P99
+  TPOT), each the mean over a workload's replicas (the paper averages its
+  rows over arrival traces).
 
 Everything here is argument marshalling and control flow; the arithmetic runs
 in the CUDA kernels behind ``ctr``.
@@ -185,3 +188,36 @@ def calibration_saturation(widths=(3, 4, 5, 6, 7), mixes=(1.0, 5 / 6, 2 / 3, 1 /
     laws = [W.TraceCfg(mix_short_thr=W.prob_to_u32_threshold(m)) for m in mixes]
     return {w: saturation_rate(laws, W.SimCfg(n_prefill=2, n_decode=w), n_req=n_req, device=device)
             for w in widths}
+
+
+def policy_table(wl, n_replicas: int = None, n_req: int = None, policies=None, const_set=None,
+                 device="cuda") -> dict:
+    """{policy name: {"goodput", "p99_ttft_s", "p99_tpot_s", "rows_failed"}}: Table 2's columns for one
+    workload, each the mean over its replicas of the per-row values (goodput = met / requests; the P99s in
+    seconds, rows without a multi-token request left out of the TPOT mean).  One trace, one simulation of
+    every policy, one goodput pass with P99 TPOT."""
+    R = n_replicas or wl.n_replicas
+    N = n_req or wl.n_req
+    pols = list(policies or wl.policies)
+    cc = const_set or wl.consts[0]
+    buf = alloc(wl.sim, R, R * len(pols), N, device)
+    run_step(wl.trace, wl.sim, [cc], pols, R, N, 0, buf)
+    tpot = torch.empty(R * len(pols), dtype=torch.int64, device=device)
+    ctr.ctr_goodput(wl.sim, buf.trace, R, len(pols), N, buf.t_first, buf.t_done, buf.met, buf.p99,
+                    p99_tpot_us=tpot)
+    torch.cuda.synchronize()
+    ok = (buf.row_status == ctr.CTR_OK).view(R, len(pols))
+    met = buf.met.view(R, len(pols)).double()
+    p99 = buf.p99.view(R, len(pols)).double()
+    tp = tpot.view(R, len(pols)).double()
+    out = {}
+    for j, pol in enumerate(pols):
+        good = ok[:, j]
+        has_tpot = good & (tp[:, j] >= 0)
+        out[W.POLICY_NAMES[pol]] = {
+            "goodput": float((met[good, j] / max(N, 1)).mean()) if good.any() else None,
+            "p99_ttft_s": float(p99[good, j].mean() / 1e6) if good.any() else None,
+            "p99_tpot_s": float(tp[has_tpot, j].mean() / 1e6) if has_tpot.any() else None,
+            "rows_failed": int((~good).sum()),
+        }
+    return out

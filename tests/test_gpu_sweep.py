@@ -182,3 +182,29 @@ def test_calibration_sweep_batched(orc):
                     assert st_b[r * 3 + b] == o["status"]
                     if o["status"] == 0:
                         assert int(h_b[r * 3 + b]) == o["hash"]
+
+
+def test_policy_table_is_the_mean_of_oracle_rows(orc):
+    """Table 2's columns per policy: the mean over replicas of each row's goodput, P99 TTFT and P99 TPOT,
+    every row recomputed by the oracle from the oracle's own simulation of the same trace."""
+    from paper_2609_16206_gb300 import ctr, sweep
+    need_gpu()
+    wl = W.replica_sweep(n_replicas=3, n_req=3000)
+    table = sweep.policy_table(wl)
+    tr = ctr.empty_requests(wl.n_replicas, wl.n_req, "cuda")
+    ctr.ctr_gen_trace(wl.trace, wl.n_replicas, 0, wl.n_req, tr)
+    torch.cuda.synchronize()
+    for pol in wl.policies:
+        gp, ttft, tpot = [], [], []
+        for r in range(wl.n_replicas):
+            trh = host_trace(tr, r)
+            o = orc.simulate(wl.sim, wl.consts[0], pol, trh)
+            met, p99 = orc.goodput(wl.sim, trh, o["t_first_us"], o["t_done_us"])
+            gp.append(met / wl.n_req)
+            ttft.append(p99 / 1e6)
+            tpot.append(orc.p99_tpot(trh, o["t_first_us"], o["t_done_us"]) / 1e6)
+        row = table[W.POLICY_NAMES[pol]]
+        assert row["rows_failed"] == 0
+        assert row["goodput"] == pytest.approx(np.mean(gp), rel=1e-12)
+        assert row["p99_ttft_s"] == pytest.approx(np.mean(ttft), rel=1e-12)
+        assert row["p99_tpot_s"] == pytest.approx(np.mean(tpot), rel=1e-12)
