@@ -311,7 +311,8 @@ __global__ void __launch_bounds__(kThreads, 2) goodput_kernel(const GoodputParam
     }
 }
 
-// P99 TPOT per row (Table 2): one block per row.  A request with o >= 2
+// P99 TPOT per row (Table 2): one block per row, each thread taking two
+// requests per pass with all their loads issued first.  A request with o >= 2
 // output tokens has TPOT = (t_done - t_first) / (o - 1) rounded toward zero
 // (the floor, as t_done >= t_first); one-token requests have none.  Pass 1
 // counts the row's M such requests and histograms their TPOTs over the same
@@ -349,15 +350,25 @@ __global__ void __launch_bounds__(kThreads, 2) tpot_kernel(const GoodputParams P
         __syncthreads();
         int32_t m = 0;
         int32_t wide = 0;  // a decode time outside [0, 2^32)
-        for (int64_t k = tid; k < n; k += kThreads) {
-            const int32_t o = __ldg(&P.trace.true_out[tb + k]);
-            if (o < 2) continue;
-            m += 1;
-            const int64_t d = __ldg(&P.t_done[ob + k]) - __ldg(&P.t_first[ob + k]);
-            if ((uint64_t)d < (uint64_t(1) << 32)) {
-                atomicAdd(&hist[log_bin((uint32_t)d / (uint32_t)(o - 1))], 1u);
-            } else {
-                wide = 1;
+        for (int64_t k0 = tid; k0 < n; k0 += 2 * kThreads) {  // two requests per thread, loads first
+            int32_t o[2];
+            int64_t d[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int64_t k = k0 + u * kThreads < n ? k0 + u * kThreads : k0;
+                o[u] = __ldg(&P.trace.true_out[tb + k]);
+                d[u] = __ldg(&P.t_done[ob + k]) - __ldg(&P.t_first[ob + k]);
+            }
+            if (k0 + kThreads >= n) o[1] = 0;  // past the end: no request
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                if (o[u] < 2) continue;
+                m += 1;
+                if ((uint64_t)d[u] < (uint64_t(1) << 32)) {
+                    atomicAdd(&hist[log_bin((uint32_t)d[u] / (uint32_t)(o[u] - 1))], 1u);
+                } else {
+                    wide = 1;
+                }
             }
         }
         const int32_t M = block_reduce<int32_t>(m, 0, [](int32_t a, int32_t b) { return a + b; },
@@ -374,11 +385,24 @@ __global__ void __launch_bounds__(kThreads, 2) tpot_kernel(const GoodputParams P
             find_rank_bin(hist, kLogBins, rank, S.pick, S.wsum);  // its barriers also publish n_cand
             const uint32_t B = S.pick[0];
             const int64_t r_in = rank - (int64_t)S.pick[1];
-            for (int64_t k = tid; k < n; k += kThreads) {
-                uint32_t v;
-                if (tpot32_of(P, tb, ob, k, v) && log_bin(v) == B) {
-                    const uint32_t i = atomicAdd(&S.n_cand, 1u);
-                    if (i < (uint32_t)kCand) S.cand_v[i] = (int64_t)v;
+            for (int64_t k0 = tid; k0 < n; k0 += 2 * kThreads) {
+                int32_t o[2];
+                uint32_t d[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int64_t k = k0 + u * kThreads < n ? k0 + u * kThreads : k0;
+                    o[u] = __ldg(&P.trace.true_out[tb + k]);
+                    d[u] = (uint32_t)(__ldg(&P.t_done[ob + k]) - __ldg(&P.t_first[ob + k]));
+                }
+                if (k0 + kThreads >= n) o[1] = 0;
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (o[u] < 2) continue;
+                    const uint32_t v = d[u] / (uint32_t)(o[u] - 1);
+                    if (log_bin(v) == B) {
+                        const uint32_t i = atomicAdd(&S.n_cand, 1u);
+                        if (i < (uint32_t)kCand) S.cand_v[i] = (int64_t)v;
+                    }
                 }
             }
             __syncthreads();
