@@ -172,3 +172,16 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     assert not t.is_alive(), "loading a missing library blocked"
     assert "err" in out and "is missing" in str(out["err"])
     assert ctr.ctr_strerror(ctr.CTR_EINVAL) == "libctr.so not loaded"
+
+
+def test_binding_switches_between_the_two_libraries():
+    """ctr.use_library loads the bounds-checked twin and back (no device calls)."""
+    from paper_2609_16206_gb300 import build, ctr
+    build.build()
+    checked = build.build(checked=True)
+    before = ctr.use_library(checked)
+    try:
+        assert ctr.ctr_bounds_checked() == 1 and ctr.ctr_abi_version() == 8
+    finally:
+        ctr.use_library(before)
+    assert ctr.LIB_PATH == before and ctr.ctr_bounds_checked() == 0
