@@ -16,6 +16,10 @@
 * ``policy_table`` -- Table 2's columns per policy (goodput, P99 TTFT, P99
   TPOT), each the mean over a workload's replicas (the paper averages its
   rows over arrival traces).
+* ``resumable_sweep`` / ``read_journal`` -- a sweep in replica chunks with a
+  per-chunk journal, so that a killed sweep restarts where it stopped (the
+  paper journals every run per request and resumes it, sec. IV-A); every row
+  depends on its seeds alone, so a resumed sweep equals an uninterrupted one.
 
 Everything here is argument marshalling and control flow; the arithmetic runs
 in the CUDA kernels behind ``ctr``.
@@ -23,7 +27,11 @@ in the CUDA kernels behind ``ctr``.
 from __future__ import annotations
 
 import dataclasses
+import hashlib
+import json
+import os
 
+import numpy as np
 import torch
 
 from . import ctr
@@ -221,3 +229,104 @@ def policy_table(wl, n_replicas: int = None, n_req: int = None, policies=None, c
             "rows_failed": int((~good).sum()),
         }
     return out
+
+
+# ---------------------------------------------------------------- resumable sweeps
+JOURNAL_VERSION = 1
+_U64 = (1 << 64) - 1
+RESULT_FIELDS = ("row_hash", "row_status", "met", "p99_ttft_us")
+
+
+def sweep_fingerprint(wl, const_sets, policies, chunk: int) -> str:
+    """A digest of everything that determines a sweep's rows and chunking (a journal of another sweep is refused)."""
+    d = {"version": JOURNAL_VERSION, "trace": dataclasses.asdict(wl.trace), "sim": dataclasses.asdict(wl.sim),
+         "consts": [dataclasses.asdict(c) for c in const_sets], "policies": [int(p) for p in policies],
+         "n_replicas": int(wl.n_replicas), "n_req": int(wl.n_req), "chunk": int(chunk)}
+    return hashlib.sha256(json.dumps(d, sort_keys=True).encode()).hexdigest()
+
+
+def read_journal(path: str, fingerprint: str, repair: bool = False) -> dict:
+    """{replica offset: record} of the chunks in a journal (one JSON line per finished chunk).  A last line
+    without its newline is an append that was cut short: it is ignored (and, with repair, cut off the file so
+    the next append starts on a line of its own).  Any other unreadable line, or a line of another sweep,
+    raises ValueError."""
+    done = {}
+    if not os.path.exists(path):
+        return done
+    with open(path, "rb") as f:
+        data = f.read()
+    good_end, pos = 0, 0
+    while pos < len(data):
+        nl = data.find(b"\n", pos)
+        if nl < 0:  # the torn tail of an interrupted append
+            break
+        line = data[pos:nl]
+        pos = nl + 1
+        if line.strip():
+            try:
+                rec = json.loads(line)
+            except json.JSONDecodeError as e:
+                raise ValueError(f"{path}: unreadable journal line ending at byte {nl}") from e
+            if rec.get("fingerprint") != fingerprint:
+                raise ValueError(f"{path} is the journal of another sweep")
+            done[int(rec["offset"])] = rec
+        good_end = pos
+    if repair and good_end < len(data):
+        with open(path, "r+b") as f:
+            f.truncate(good_end)
+    return done
+
+
+def _gpu_chunk_runner(wl, const_sets, policies, chunk: int, device):
+    """run(offset, count): trace, simulation and goodput of replicas [offset, offset + count) on the GPU."""
+    per = len(const_sets) * len(policies)
+    buf = alloc(wl.sim, chunk, chunk * per, wl.n_req, device)
+
+    def run(off: int, cnt: int) -> dict:
+        rows = cnt * per
+        trace = {k: v[:cnt] for k, v in buf.trace.items()}
+        ctr.ctr_gen_trace(wl.trace, cnt, off, wl.n_req, trace)
+        ctr.ctr_simulate(wl.sim, const_sets, policies, trace, cnt, wl.n_req, buf.t_first[:rows], buf.t_done[:rows],
+                         buf.row_hash[:rows], buf.row_status[:rows], buf.workspace, met_count=buf.met[:rows],
+                         p99_ttft_us=buf.p99[:rows])
+        torch.cuda.synchronize()
+        return {"row_hash": [int(x) & _U64 for x in buf.row_hash[:rows].tolist()],
+                "row_status": buf.row_status[:rows].tolist(), "met": buf.met[:rows].tolist(),
+                "p99_ttft_us": buf.p99[:rows].tolist()}
+    return run
+
+
+def resumable_sweep(wl, journal: str, chunk: int = 256, const_sets=None, policies=None, device="cuda",
+                    max_chunks: int = None, run_chunk=None):
+    """The rows of workload `wl` (replica x constant set x policy) simulated in chunks of `chunk` replicas.
+    Each finished chunk's per-row checksum, status, met count and P99 TTFT go to `journal` as one JSON line,
+    flushed and fsynced, before the next chunk starts; chunks already in the journal are not simulated again.
+    So a sweep that is killed (a lost rank, a pre-empted job) restarts where it stopped, and its rows equal
+    those of one uninterrupted run: a row is a function of its replica's seeds alone.  `max_chunks` stops
+    after that many new chunks.  Returns {field: numpy array over all rows, replica-major} once every chunk
+    is journaled, else None.  `run_chunk(offset, count) -> {field: list}` replaces the GPU runner (tests)."""
+    const_sets = list(const_sets or wl.consts)
+    policies = list(policies or wl.policies)
+    if chunk < 1:
+        raise ValueError("chunk must be positive")
+    fp = sweep_fingerprint(wl, const_sets, policies, chunk)
+    done = read_journal(journal, fp, repair=True)
+    offsets = list(range(0, wl.n_replicas, chunk))
+    todo = [o for o in offsets if o not in done]
+    if max_chunks is not None:
+        todo = todo[:max_chunks]
+    if todo:
+        run = run_chunk or _gpu_chunk_runner(wl, const_sets, policies, chunk, device)
+        for off in todo:
+            cnt = min(chunk, wl.n_replicas - off)
+            rec = {"fingerprint": fp, "offset": off, "count": cnt}
+            rec.update(run(off, cnt))
+            with open(journal, "a") as f:
+                f.write(json.dumps(rec) + "\n")
+                f.flush()
+                os.fsync(f.fileno())
+            done[off] = rec
+    if any(o not in done for o in offsets):
+        return None
+    return {k: np.concatenate([np.asarray(done[o][k], dtype=np.uint64 if k == "row_hash" else np.int64)
+                               for o in offsets]) for k in RESULT_FIELDS}

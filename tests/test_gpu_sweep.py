@@ -208,3 +208,27 @@ def test_policy_table_is_the_mean_of_oracle_rows(orc):
         assert row["goodput"] == pytest.approx(np.mean(gp), rel=1e-12)
         assert row["p99_ttft_s"] == pytest.approx(np.mean(ttft), rel=1e-12)
         assert row["p99_tpot_s"] == pytest.approx(np.mean(tpot), rel=1e-12)
+
+
+def test_resumable_sweep_equals_one_shot(orc, tmp_path):
+    """A sweep stopped after its first chunk and resumed from its journal gives, row for row, the
+    checksums, statuses, met counts and P99 TTFTs of one launch over all replicas (chunks of 3, 3 and 1
+    replicas from their own trace offsets)."""
+    from paper_2609_16206_gb300 import ctr, sweep
+    need_gpu()
+    wl = W.replica_sweep(n_replicas=7, n_req=1500)
+    j = str(tmp_path / "journal")
+    assert sweep.resumable_sweep(wl, j, chunk=3, max_chunks=1) is None
+    res = sweep.resumable_sweep(wl, j, chunk=3)
+    rows = wl.n_replicas * len(wl.policies)
+    buf = sweep.alloc(wl.sim, wl.n_replicas, rows, wl.n_req, "cuda")
+    sweep.run_step(wl.trace, wl.sim, wl.consts, list(wl.policies), wl.n_replicas, wl.n_req, 0, buf)
+    torch.cuda.synchronize()
+    assert np.array_equal(res["row_hash"], buf.row_hash.cpu().numpy().astype(np.uint64))
+    assert np.array_equal(res["row_status"], buf.row_status.cpu().numpy())
+    assert np.array_equal(res["met"], buf.met.cpu().numpy())
+    assert np.array_equal(res["p99_ttft_us"], buf.p99.cpu().numpy())
+    assert (res["row_status"] == ctr.CTR_OK).all()
+    trh = host_trace(buf.trace, 6)  # the last chunk's replica against the oracle
+    for j_, pol in enumerate(wl.policies):
+        assert int(res["row_hash"][6 * len(wl.policies) + j_]) == orc.simulate(wl.sim, wl.consts[0], pol, trh)["hash"]
