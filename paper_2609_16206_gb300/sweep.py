@@ -328,5 +328,8 @@ def resumable_sweep(wl, journal: str, chunk: int = 256, const_sets=None, policie
             done[off] = rec
     if any(o not in done for o in offsets):
         return None
-    return {k: np.concatenate([np.asarray(done[o][k], dtype=np.uint64 if k == "row_hash" else np.int64)
-                               for o in offsets]) for k in RESULT_FIELDS}
+    out = {}
+    for k in RESULT_FIELDS:
+        dt = np.uint64 if k == "row_hash" else np.int64
+        out[k] = np.concatenate([np.zeros(0, dt)] + [np.asarray(done[o][k], dtype=dt) for o in offsets])
+    return out

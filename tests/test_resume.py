@@ -103,3 +103,10 @@ def test_corrupt_line_inside_the_journal_raises(tmp_path):
     open(j, "w").write("{not json}\n" + text)
     with pytest.raises(ValueError):
         sweep.resumable_sweep(WL, str(j), chunk=5, run_chunk=Runner())
+
+
+def test_no_replicas(tmp_path):
+    empty = W.replica_sweep(n_replicas=0, n_req=100)
+    run = Runner()
+    res = sweep.resumable_sweep(empty, str(tmp_path / "j"), chunk=3, run_chunk=run)
+    assert run.calls == [] and all(res[k].size == 0 for k in sweep.RESULT_FIELDS)
