@@ -18,7 +18,7 @@
   rows over arrival traces).
 * ``resumable_sweep`` / ``read_journal`` -- a sweep in replica chunks with a
   per-chunk journal, so that a killed sweep restarts where it stopped (the
-  paper journals every run per request and resumes it, sec. IV-A); every row
+  paper journals every run per request and resumes it, sec. IV-B); every row
   depends on its seeds alone, so a resumed sweep equals an uninterrupted one.
 
 Everything here is argument marshalling and control flow; the arithmetic runs
